@@ -1,0 +1,6 @@
+"""fp64 CPU oracle of the SA sketching step (test infrastructure only).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU baseline /
+reference legs may import this package; the product path never does.
+"""
+from .sa_oracle import affinity, proto_softmax, sa_backward, sa_forward  # noqa: F401

@@ -1,0 +1,110 @@
+"""fp64 CPU oracle of the Sketch Attention (SA) sketching step.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import, call or
+execute this module: only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` use it.  It shares
+no code with the CUDA library; the two meet only in the seeded inputs drawn by
+``paper_2609_08443_gb300.workloads`` (which holds none of the arithmetic).
+
+What it computes (paper Sec. 3.1, equations for S, A and the sketch
+``eq:sa-sketch``; the same three steps are listed in App. B):
+
+  per user b (rows cu[b]..cu[b+1] of the packed K, V) and head h:
+    S[j, i]  = scale * <Q[h, j, :], K_b[i, h, :]>          P x L_b   (affinity)
+    A[:, i]  = softmax over the prototype axis j of S[:, i]          (prototype-wise
+               normalisation: every token spreads unit mass over the P prototypes)
+    O[b, h]  = A @ V_b[:, h, :]                             P x d     (sketch)
+
+The paper normalises nothing further: the sketch is the plain weighted sum
+over tokens (Sec. 3.1, "Sketch construction").  Heads are independent copies
+of the single-head SA of the paper.  ``scale`` is passed in; the paper uses
+1/sqrt(d) with d the SA width.
+
+The paper prints no backward pass; it states only that the sketch is fully
+differentiable and trained end to end (Sec. 3.1, App. F).  The gradient below
+is the chain rule of the three forward steps with upstream G = dL/dO[b, h]:
+    dV_b   = A^T G                                   (L_b x d)
+    dA     = G V_b^T                                 (P x L_b)
+    dS     = A * (dA - 1 colsum(A * dA))   (softmax Jacobian along the prototype axis)
+    dK_b   = scale * dS^T Q[h]                       (L_b x d)
+    dQ[h] += scale * dS K_b    summed over ALL users, because the prototypes are
+                               shared globally (Sec. 3.1)
+
+All arithmetic is float64; bf16 inputs arrive already widened exactly.
+Parity pins for both functions live in ``tests/test_oracle.py`` (brute force
+in 50-digit arithmetic, closed forms, invariants, finite differences).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def _user_slices(cu_seqlens):
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    return [(int(cu[b]), int(cu[b + 1])) for b in range(cu.size - 1)]
+
+
+def affinity(Qh, Kbh, scale):
+    """S = scale * Q K^T for one (user, head): P x L (Sec. 3.1, affinity S)."""
+    return scale * (Qh @ Kbh.T)
+
+
+def proto_softmax(S):
+    """Softmax along axis 0 (the prototype axis) of a P x L score matrix.
+
+    The per-column max is subtracted first; in exact arithmetic this shift
+    cancels (Sec. 3.1, A = softmax_proto(S)).
+    """
+    m = S.max(axis=0, keepdims=True)
+    e = np.exp(S - m)
+    return e / e.sum(axis=0, keepdims=True)
+
+
+def sa_forward(K, V, cu_seqlens, Q, scale, with_lse=False):
+    """Sketch O[B, H, P, d] (and optionally per-token log-sum-exp lse[N, H]).
+
+    K, V: [N, H, d] float64;  Q: [H, P, d] float64;  cu_seqlens: [B + 1].
+    A user with no tokens gets an all-zero sketch (empty sum).
+    """
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Q = np.asarray(Q, dtype=np.float64)
+    H, P, d = Q.shape
+    sl = _user_slices(cu_seqlens)
+    O = np.zeros((len(sl), H, P, d))
+    lse = np.zeros((K.shape[0], H))
+    for b, (t0, t1) in enumerate(sl):
+        if t1 == t0:
+            continue
+        for h in range(H):
+            S = affinity(Q[h], K[t0:t1, h, :], scale)
+            A = proto_softmax(S)
+            O[b, h] = A @ V[t0:t1, h, :]
+            if with_lse:
+                m = S.max(axis=0)
+                lse[t0:t1, h] = m + np.log(np.exp(S - m).sum(axis=0))
+    return (O, lse) if with_lse else O
+
+
+def sa_backward(K, V, cu_seqlens, Q, scale, dO):
+    """Gradients (dK [N,H,d], dV [N,H,d], dQ [H,P,d]) of L = sum(dO * O)."""
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Q = np.asarray(Q, dtype=np.float64)
+    dO = np.asarray(dO, dtype=np.float64)
+    H, P, d = Q.shape
+    dK = np.zeros_like(K)
+    dV = np.zeros_like(V)
+    dQ = np.zeros_like(Q)
+    for b, (t0, t1) in enumerate(_user_slices(cu_seqlens)):
+        if t1 == t0:
+            continue
+        for h in range(H):
+            Kb, Vb, G = K[t0:t1, h, :], V[t0:t1, h, :], dO[b, h]
+            A = proto_softmax(affinity(Q[h], Kb, scale))
+            dV[t0:t1, h, :] = A.T @ G
+            dA = G @ Vb.T
+            dS = A * (dA - (A * dA).sum(axis=0, keepdims=True))
+            dK[t0:t1, h, :] = scale * (dS.T @ Q[h])
+            dQ[h] += scale * (dS @ Kb)
+    return dK, dV, dQ

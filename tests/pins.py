@@ -1,0 +1,301 @@
+"""Pins of the SA oracle against facts the paper and mathematics fix.
+
+Every ``pin_*`` takes the forward and backward functions under test (with the
+signatures of ``oracle.sa_forward`` / ``oracle.sa_backward``) and raises
+AssertionError when they disagree with:
+
+  * a 50-digit brute-force evaluation of the paper's definition (Sec. 3.1:
+    affinity S, prototype-wise softmax A, sketch A X), written as plain loops
+    with no stabilising shift;
+  * 50-digit central finite differences of that brute force (for the gradient,
+    which the paper does not print);
+  * the conservation law sum_j A[j, i] = 1 (Sec. 3.1, App. C): with V = 1 every
+    sketch column sums to the user's history length;
+  * closed forms: equal prototypes give uniform weights 1/P; P = 1 is sum
+    pooling; L = 1 is one softmax (scipy.special.softmax); a huge scale gives
+    a hard arg-max assignment;
+  * invariances: token order within a user (SA has no positional term), ragged
+    batch = users run alone, heads independent, linear in V, common shift of
+    all prototypes; and the gradient facts those imply (sum_j dQ[h, j] = 0,
+    dK = 0 for equal prototypes, dV_i = g when every row of G equals g).
+
+``tests/test_oracle_mutants.py`` plants plausible mistakes in copies of the
+oracle and checks that each is caught by at least one pin.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _rand_problem(seed, lens, H, P, d, q_std=1.0):
+    r = _rng(seed)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    N = int(cu[-1])
+    K = r.standard_normal((N, H, d))
+    V = r.standard_normal((N, H, d))
+    Q = q_std * r.standard_normal((H, P, d))
+    dO = r.standard_normal((len(lens), H, P, d))
+    return K, V, cu, Q, dO
+
+
+def _close(a, b, rtol, what):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    assert a.shape == b.shape, f"{what}: shape {a.shape} != {b.shape}"
+    scale = max(1.0, float(np.max(np.abs(b)))) if b.size else 1.0
+    err = float(np.max(np.abs(a - b))) if a.size else 0.0
+    assert err <= rtol * scale, f"{what}: max err {err:.3e} > {rtol:.1e} * {scale:.3e}"
+
+
+# ----------------------------------------------------------- brute force
+
+def _mp_forward(K, V, cu, Q, scale, mp):
+    """Plain-loop evaluation of O = softmax_proto(S) X in mpmath (no shift)."""
+    H, P, d = len(Q), len(Q[0]), len(Q[0][0])
+    B = len(cu) - 1
+    O = [[[[mp.mpf(0)] * d for _ in range(P)] for _ in range(H)] for _ in range(B)]
+    for b in range(B):
+        for h in range(H):
+            for i in range(int(cu[b]), int(cu[b + 1])):
+                ex = []
+                for j in range(P):
+                    s = mp.mpf(0)
+                    for c in range(d):
+                        s += mp.mpf(Q[h][j][c]) * mp.mpf(K[i][h][c])
+                    ex.append(mp.exp(mp.mpf(scale) * s))
+                z = mp.fsum(ex)
+                for j in range(P):
+                    a = ex[j] / z
+                    for c in range(d):
+                        O[b][h][j][c] += a * mp.mpf(V[i][h][c])
+    return O
+
+
+def _mp_loss(K, V, cu, Q, scale, dO, mp):
+    O = _mp_forward(K, V, cu, Q, scale, mp)
+    tot = mp.mpf(0)
+    B, H, P, d = dO.shape
+    for b in range(B):
+        for h in range(H):
+            for j in range(P):
+                for c in range(d):
+                    tot += mp.mpf(dO[b, h, j, c]) * O[b][h][j][c]
+    return tot
+
+
+def pin_bruteforce_forward(fwd, bwd=None):
+    import mpmath as mp
+    mp.mp.dps = 50
+    K, V, cu, Q, _ = _rand_problem(1, [3, 0, 2, 1], H=2, P=3, d=2)
+    scale = 0.7
+    ref = _mp_forward(K.tolist(), V.tolist(), cu, Q.tolist(), scale, mp)
+    got = fwd(K, V, cu, Q, scale)
+    refa = np.array([[[[float(x) for x in row] for row in hh] for hh in bb] for bb in ref])
+    _close(got, refa, 1e-13, "brute-force sketch")
+
+
+def pin_bruteforce_lse(fwd, bwd=None):
+    import mpmath as mp
+    mp.mp.dps = 50
+    K, V, cu, Q, _ = _rand_problem(2, [2, 3], H=2, P=4, d=3)
+    scale = 1.3
+    _, lse = fwd(K, V, cu, Q, scale, with_lse=True)
+    for i in range(K.shape[0]):
+        for h in range(2):
+            z = mp.fsum(mp.exp(mp.mpf(scale) * mp.fsum(mp.mpf(Q[h, j, c]) * mp.mpf(K[i, h, c])
+                                                     for c in range(3))) for j in range(4))
+            assert abs(float(mp.log(z)) - lse[i, h]) < 1e-12, "lse"
+
+
+def pin_bruteforce_gradients(fwd, bwd):
+    """50-digit central differences of sum(dO * O) against the backward."""
+    import mpmath as mp
+    mp.mp.dps = 50
+    K, V, cu, Q, dO = _rand_problem(3, [2, 3], H=2, P=3, d=2)
+    scale = 0.9
+    dK, dV, dQ = bwd(K, V, cu, Q, scale, dO)
+    eps = mp.mpf("1e-20")
+
+    def fd(arr_name, idx):
+        base = {"K": K.tolist(), "V": V.tolist(), "Q": Q.tolist()}
+
+        def with_delta(delta):
+            a = [list(map(list, x)) for x in base[arr_name]]
+            i, j, k = idx
+            a[i][j][k] = mp.mpf(a[i][j][k]) + delta
+            args = dict(base)
+            args[arr_name] = a
+            return _mp_loss(args["K"], args["V"], cu, args["Q"], scale, dO, mp)
+
+        return float((with_delta(eps) - with_delta(-eps)) / (2 * eps))
+
+    for name, grad in (("K", dK), ("V", dV), ("Q", dQ)):
+        for idx in np.ndindex(*grad.shape):
+            ref = fd(name, idx)
+            assert abs(grad[idx] - ref) <= 1e-11 * max(1.0, abs(ref)), \
+                f"d{name}{idx}: {grad[idx]} vs finite difference {ref}"
+
+
+# ------------------------------------------------------------ invariants
+
+def pin_conservation(fwd, bwd=None):
+    lens = [5, 1, 0, 17]
+    K, V, cu, Q, _ = _rand_problem(4, lens, H=3, P=7, d=4)
+    O = fwd(K, np.ones_like(V), cu, Q, 0.5)
+    for b, L in enumerate(lens):
+        _close(O[b].sum(axis=1), np.full((3, 4), float(L)), 1e-13, "column sums = L_b")
+
+
+def pin_equal_prototypes(fwd, bwd):
+    lens = [6, 3]
+    K, V, cu, Q, dO = _rand_problem(5, lens, H=2, P=5, d=3)
+    Q[:] = Q[:, :1, :]  # every prototype row identical
+    O = fwd(K, V, cu, Q, 0.8)
+    for b in range(2):
+        t0, t1 = cu[b], cu[b + 1]
+        mean = V[t0:t1].sum(axis=0) / 5.0  # (H, d)
+        _close(O[b], np.repeat(mean[:, None, :], 5, axis=1), 1e-13, "uniform weights")
+    dK, _, _ = bwd(K, V, cu, Q, 0.8, dO)
+    _close(dK, np.zeros_like(dK), 1e-13, "dK = 0 for equal prototypes")
+
+
+def pin_single_prototype(fwd, bwd=None):
+    lens = [4, 9]
+    K, V, cu, Q, _ = _rand_problem(6, lens, H=2, P=1, d=3)
+    O = fwd(K, V, cu, Q, 1.1)
+    for b in range(2):
+        _close(O[b][:, 0, :], V[cu[b]:cu[b + 1]].sum(axis=0), 1e-13, "P=1 sum pooling")
+
+
+def pin_single_token(fwd, bwd=None):
+    from scipy.special import softmax
+    K, V, cu, Q, _ = _rand_problem(7, [1], H=2, P=6, d=4)
+    O = fwd(K, V, cu, Q, 0.3)
+    for h in range(2):
+        w = softmax(0.3 * (Q[h] @ K[0, h]))
+        _close(O[0, h], np.outer(w, V[0, h]), 1e-13, "L=1 softmax")
+
+
+def pin_hard_assignment(fwd, bwd=None):
+    r = _rng(8)
+    P, d, L = 4, 4, 12
+    Q = np.eye(P, d)[None] * 1.0
+    # each token points mostly at one prototype; the margin is large
+    owner = r.integers(0, P, size=L)
+    K = (np.eye(P, d)[owner] * 3.0 + 0.1 * r.standard_normal((L, d)))[:, None, :]
+    V = r.standard_normal((L, 1, d))
+    cu = np.array([0, L])
+    O = fwd(K, V, cu, Q, 200.0)
+    ref = np.zeros((P, d))
+    for i in range(L):
+        ref[owner[i]] += V[i, 0]
+    _close(O[0, 0], ref, 1e-10, "hard assignment")
+
+
+def pin_permutation(fwd, bwd):
+    lens = [7, 5]
+    K, V, cu, Q, dO = _rand_problem(9, lens, H=2, P=4, d=3)
+    perm = np.concatenate([np.random.default_rng(1).permutation(7),
+                           7 + np.random.default_rng(2).permutation(5)])
+    O1 = fwd(K, V, cu, Q, 0.6)
+    O2 = fwd(K[perm], V[perm], cu, Q, 0.6)
+    _close(O2, O1, 1e-13, "token order")
+    g1 = bwd(K, V, cu, Q, 0.6, dO)
+    g2 = bwd(K[perm], V[perm], cu, Q, 0.6, dO)
+    _close(g2[0], g1[0][perm], 1e-13, "dK permuted")
+    _close(g2[1], g1[1][perm], 1e-13, "dV permuted")
+    _close(g2[2], g1[2], 1e-12, "dQ order")
+
+
+def pin_ragged_batch(fwd, bwd):
+    lens = [3, 0, 8, 1]
+    K, V, cu, Q, dO = _rand_problem(10, lens, H=2, P=5, d=3)
+    O = fwd(K, V, cu, Q, 0.4)
+    dK, dV, dQ = bwd(K, V, cu, Q, 0.4, dO)
+    dQ_sum = np.zeros_like(dQ)
+    for b in range(4):
+        t0, t1 = cu[b], cu[b + 1]
+        one = np.array([0, t1 - t0])
+        _close(O[b:b + 1], fwd(K[t0:t1], V[t0:t1], one, Q, 0.4), 1e-13, "batch vs alone")
+        gk, gv, gq = bwd(K[t0:t1], V[t0:t1], one, Q, 0.4, dO[b:b + 1])
+        _close(dK[t0:t1], gk, 1e-13, "dK batch vs alone")
+        _close(dV[t0:t1], gv, 1e-13, "dV batch vs alone")
+        dQ_sum += gq
+    _close(dQ, dQ_sum, 1e-12, "dQ is the sum over users")
+
+
+def pin_heads_independent(fwd, bwd=None):
+    lens = [6]
+    K, V, cu, Q, _ = _rand_problem(11, lens, H=3, P=4, d=2)
+    O = fwd(K, V, cu, Q, 0.7)
+    K2, V2, Q2 = K.copy(), V.copy(), Q.copy()
+    K2[:, 1] += 1.0
+    V2[:, 1] *= -2.0
+    Q2[1] = 0.0
+    O2 = fwd(K2, V2, cu, Q2, 0.7)
+    _close(O2[:, [0, 2]], O[:, [0, 2]], 1e-13, "other heads untouched")
+
+
+def pin_linear_in_v(fwd, bwd=None):
+    lens = [5, 4]
+    K, V, cu, Q, _ = _rand_problem(12, lens, H=2, P=3, d=3)
+    V2 = _rng(13).standard_normal(V.shape)
+    lhs = fwd(K, 2.0 * V - 0.5 * V2, cu, Q, 0.5)
+    rhs = 2.0 * fwd(K, V, cu, Q, 0.5) - 0.5 * fwd(K, V2, cu, Q, 0.5)
+    _close(lhs, rhs, 1e-13, "linear in V")
+
+
+def pin_prototype_shift(fwd, bwd):
+    lens = [6, 2]
+    K, V, cu, Q, dO = _rand_problem(14, lens, H=2, P=5, d=3)
+    u = _rng(15).standard_normal((2, 1, 3))
+    _close(fwd(K, V, cu, Q + u, 0.9), fwd(K, V, cu, Q, 0.9), 1e-12, "common shift")
+    _, _, dQ = bwd(K, V, cu, Q, 0.9, dO)
+    _close(dQ.sum(axis=1), np.zeros((2, 3)), 1e-12, "sum_j dQ = 0")
+
+
+def pin_constant_upstream(fwd, bwd):
+    lens = [4, 3]
+    K, V, cu, Q, _ = _rand_problem(16, lens, H=2, P=6, d=3)
+    g = _rng(17).standard_normal((2, 2, 1, 3))
+    dO = np.repeat(g, 6, axis=2)
+    _, dV, _ = bwd(K, V, cu, Q, 0.5, dO)
+    for b in range(2):
+        _close(dV[cu[b]:cu[b + 1]], np.repeat(g[b, :, 0][None], lens[b], axis=0), 1e-13,
+               "dV = g")
+
+
+def pin_fd_fp64(fwd, bwd):
+    """fp64 central differences at a size brute force cannot reach."""
+    lens = [9, 4]
+    K, V, cu, Q, dO = _rand_problem(18, lens, H=2, P=8, d=5)
+    scale = 1.0 / np.sqrt(5.0)
+    dK, dV, dQ = bwd(K, V, cu, Q, scale, dO)
+    r = _rng(19)
+
+    def loss(K_, V_, Q_):
+        return float(np.sum(dO * fwd(K_, V_, cu, Q_, scale)))
+
+    for name, grad in (("K", dK), ("V", dV), ("Q", dQ)):
+        for _ in range(12):
+            idx = tuple(int(r.integers(0, s)) for s in grad.shape)
+            args = {"K": K.copy(), "V": V.copy(), "Q": Q.copy()}
+            h = 1e-6
+            args[name][idx] += h
+            lp = loss(args["K"], args["V"], args["Q"])
+            args[name][idx] -= 2 * h
+            lm = loss(args["K"], args["V"], args["Q"])
+            ref = (lp - lm) / (2 * h)
+            assert abs(grad[idx] - ref) <= 1e-6 * max(1.0, abs(ref)), f"d{name}{idx}"
+
+
+ALL_PINS = [
+    pin_bruteforce_forward, pin_bruteforce_lse, pin_bruteforce_gradients, pin_conservation,
+    pin_equal_prototypes, pin_single_prototype, pin_single_token, pin_hard_assignment,
+    pin_permutation, pin_ragged_batch, pin_heads_independent, pin_linear_in_v,
+    pin_prototype_shift, pin_constant_upstream, pin_fd_fp64,
+]

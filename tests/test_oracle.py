@@ -1,0 +1,33 @@
+"""The fp64 oracle against its pins (no GPU needed)."""
+import numpy as np
+import pytest
+
+import pins
+from oracle import sa_backward, sa_forward
+
+
+@pytest.mark.parametrize("pin", pins.ALL_PINS, ids=lambda p: p.__name__)
+def test_oracle_pin(pin):
+    if pin.__name__.startswith("pin_bruteforce"):
+        pytest.importorskip("mpmath")
+    pin(sa_forward, sa_backward)
+
+
+def test_empty_user_gives_zero_sketch_and_no_nan():
+    K = np.random.default_rng(0).standard_normal((3, 1, 4))
+    cu = np.array([0, 0, 3, 3])
+    Q = np.random.default_rng(1).standard_normal((1, 5, 4))
+    O = sa_forward(K, K, cu, Q, 0.5)
+    assert np.all(O[0] == 0) and np.all(O[2] == 0) and np.all(np.isfinite(O))
+    dK, dV, dQ = sa_backward(K, K, cu, Q, 0.5, np.ones((3, 1, 5, 4)))
+    assert np.all(np.isfinite(dK)) and np.all(np.isfinite(dQ))
+
+
+def test_large_scores_do_not_overflow():
+    # scores far above exp's fp64 range still give a valid allocation
+    K = np.full((2, 1, 2), 100.0)
+    Q = np.array([[[100.0, 100.0], [99.0, 100.0]]])
+    O, lse = sa_forward(K, np.ones_like(K), np.array([0, 2]), Q, 1.0, with_lse=True)
+    assert np.all(np.isfinite(O)) and np.allclose(O[0, 0].sum() + O[0, 0].sum(), O[0, 0].sum() * 2)
+    assert np.allclose(O[0, 0, :, 0].sum(), 2.0)
+    assert np.all(np.isfinite(lse))

@@ -1,0 +1,92 @@
+"""Plant plausible mistakes in copies of the oracle; each must fail a pin.
+
+This shows that the pins in ``pins.py`` are strong enough to catch a dropped
+term, a wrong sign, a wrong softmax axis, a missing scale or a transposed
+operand anywhere in the oracle.
+"""
+import numpy as np
+import pytest
+
+import pins
+from oracle import sa_oracle as so
+
+
+def _fwd_variant(softmax=so.proto_softmax, use_scale=True, agg_from_k=False):
+    def fwd(K, V, cu, Q, scale, with_lse=False):
+        K = np.asarray(K, float); V = np.asarray(V, float); Q = np.asarray(Q, float)
+        H, P, d = Q.shape
+        sl = so._user_slices(cu)
+        O = np.zeros((len(sl), H, P, d)); lse = np.zeros((K.shape[0], H))
+        for b, (t0, t1) in enumerate(sl):
+            if t1 == t0:
+                continue
+            for h in range(H):
+                S = (scale if use_scale else 1.0) * (Q[h] @ K[t0:t1, h].T)
+                A = softmax(S)
+                O[b, h] = A @ (K if agg_from_k else V)[t0:t1, h]
+                m = S.max(axis=0)
+                lse[t0:t1, h] = m + np.log(np.exp(S - m).sum(axis=0))
+        return (O, lse) if with_lse else O
+    return fwd
+
+
+def _bwd_variant(drop_d=False, flip=False, dk_scale=True, dq_overwrite=False, dv_transpose=False):
+    def bwd(K, V, cu, Q, scale, dO):
+        K = np.asarray(K, float); V = np.asarray(V, float); Q = np.asarray(Q, float)
+        H, P, d = Q.shape
+        dK = np.zeros_like(K); dV = np.zeros_like(V); dQ = np.zeros_like(Q)
+        for b, (t0, t1) in enumerate(so._user_slices(cu)):
+            if t1 == t0:
+                continue
+            for h in range(H):
+                Kb, Vb, G = K[t0:t1, h], V[t0:t1, h], dO[b, h]
+                A = so.proto_softmax(scale * (Q[h] @ Kb.T))
+                dV[t0:t1, h] = (A.T @ G) if not dv_transpose else (A.T @ G[::-1])
+                dA = G @ Vb.T
+                Dv = 0.0 if drop_d else (A * dA).sum(axis=0, keepdims=True)
+                dS = A * ((Dv - dA) if flip else (dA - Dv))
+                dK[t0:t1, h] = (scale if dk_scale else 1.0) * (dS.T @ Q[h])
+                if dq_overwrite:
+                    dQ[h] = scale * (dS @ Kb)
+                else:
+                    dQ[h] += scale * (dS @ Kb)
+        return dK, dV, dQ
+    return bwd
+
+
+def _token_softmax(S):
+    e = np.exp(S - S.max(axis=1, keepdims=True))
+    return e / e.sum(axis=1, keepdims=True)
+
+
+def _no_shift_sum_softmax(S):  # forgets to normalise
+    return np.exp(S - S.max(axis=0, keepdims=True))
+
+
+MUTANTS = {
+    "softmax over tokens": (_fwd_variant(softmax=_token_softmax), so.sa_backward),
+    "unnormalised weights": (_fwd_variant(softmax=_no_shift_sum_softmax), so.sa_backward),
+    "scale dropped in S": (_fwd_variant(use_scale=False), so.sa_backward),
+    "aggregates K not V": (_fwd_variant(agg_from_k=True), so.sa_backward),
+    "dS without the D term": (so.sa_forward, _bwd_variant(drop_d=True)),
+    "dS sign flipped": (so.sa_forward, _bwd_variant(flip=True)),
+    "dK without scale": (so.sa_forward, _bwd_variant(dk_scale=False)),
+    "dQ not summed over users": (so.sa_forward, _bwd_variant(dq_overwrite=True)),
+    "dV with prototypes reversed": (so.sa_forward, _bwd_variant(dv_transpose=True)),
+}
+
+CHEAP_PINS = [p for p in pins.ALL_PINS if p is not pins.pin_bruteforce_gradients]
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name):
+    fwd, bwd = MUTANTS[name]
+    caught = []
+    for pin in CHEAP_PINS:
+        if pin.__name__.startswith("pin_bruteforce"):
+            pytest.importorskip("mpmath")
+        try:
+            pin(fwd, bwd)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught, f"no pin catches the planted mistake '{name}'"
