@@ -1,0 +1,376 @@
+"""Benchmark of the SA sketching step (forward + backward) on one GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+One step = one pass of the whole hot path over the 100K-token training batch:
+sa_sketch_fwd (saving the per-token lse) then sa_sketch_bwd, on 128 users x
+100000 tokens, H=8 heads, d=128, P=512 prototypes, bf16 inputs with fp32
+accumulation; K, V ~ N(0,1), Q ~ N(0, 0.02), dsketch ~ N(0,1), seeded.
+Inputs (52 GB of K and V) are far larger than L2, so no flush is needed.
+
+Prints ONE JSON line (rank 0).  `value` is sketched tokens/s of the whole job
+(tokens = sum of user lengths; every head included).  Under torchrun each rank
+runs its own full batch (weak scaling, no collective on the data path; the
+timing is the max over ranks).  `--impl reference` times the fp64 CPU oracle
+on a bounded sample of the same workload on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_08443_gb300 import roofline as rf  # noqa: E402
+from paper_2609_08443_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "SA sketched tokens/sec fwd and fwd+bwd at 100K/user; % of roofline"
+CONFIG_ID = 4
+E2E_USERS = 16
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def workload_config(spec, lens):
+    return {"workload": "SA sketch training step (fwd+bwd), 100K tokens/user",
+            "users": int(lens.size), "tokens_per_user": int(lens[0]), "tokens": int(lens.sum()),
+            "heads": spec.H, "d": spec.d, "prototypes": spec.P, "inputs": "bf16 K,V,Q; fp32 accumulate",
+            "l2": "inputs larger than L2 (K+V = %.1f GB per step), no flush" % (
+                2 * lens.sum() * spec.H * spec.d * 2 / 1e9),
+            "q_std": spec.q_std, "seed": spec.seed}
+
+
+# ------------------------------------------------------------ clocks sampling
+
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_bench_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------- oracle timing
+
+def oracle_sample(spec, budget_s=20.0, max_heads=None):
+    """Time the fp64 oracle (fwd+bwd) on one user of the workload, head by head,
+    until about ``budget_s`` of CPU work; returns tokens/s scaled to all heads."""
+    from oracle import sa_backward, sa_forward
+
+    L = int(wl.lengths(spec)[0])
+    rng = np.random.default_rng(0)
+    Q = (spec.q_std * rng.standard_normal((1, spec.P, spec.d))).astype(np.float32).astype(np.float64)
+    cu = np.array([0, L])
+    heads = 0
+    t_tot = 0.0
+    max_heads = max_heads or spec.H
+    while heads < max_heads and (t_tot < budget_s or heads == 0):
+        K = wl.bf16_bits_to_f64(wl.f32_to_bf16_bits(rng.standard_normal((L, 1, spec.d), dtype=np.float32)))
+        V = wl.bf16_bits_to_f64(wl.f32_to_bf16_bits(rng.standard_normal((L, 1, spec.d), dtype=np.float32)))
+        G = rng.standard_normal((1, 1, spec.P, spec.d))
+        t0 = time.perf_counter()
+        sa_forward(K, V, cu, Q, spec.scale, with_lse=True)
+        sa_backward(K, V, cu, Q, spec.scale, G)
+        t_tot += time.perf_counter() - t0
+        heads += 1
+    tokens_equiv = L * heads / spec.H
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {"value": tokens_equiv / t_tot, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"fp64 numpy oracle fwd+bwd on 1 user x {heads} of {spec.H} heads x {L} tokens "
+                      f"(P={spec.P}, d={spec.d}); {t_tot:.1f} s; numpy/BLAS threads on {cores} host cores",
+            "seconds": t_tot}
+
+
+def run_reference(args, spec, lens):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    step_times = []
+    info = None
+    for s in range(args.warmup + args.steps):
+        info = oracle_sample(spec, budget_s=0.0, max_heads=1)
+        if s >= args.warmup:
+            step_times.append(info["seconds"])
+    t = sum(step_times)
+    L = int(lens[0])
+    tokens_equiv = L / spec.H * len(step_times)
+    value = tokens_equiv / t
+    cpu = {"value": value, "unit": "tokens/s", "cores": info["cores"], "kind": "oracle",
+           "sample": f"each step: fp64 oracle fwd+bwd on 1 user x 1 of {spec.H} heads x {L} tokens"}
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * t / len(step_times), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": workload_config(spec, lens),
+            "cpu_baseline": cpu,
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------- GPU arm
+
+def run_ours(args, spec, lens):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_08443_gb300 import binding
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    binding.load()
+    pk = peaks()
+
+    data = wl.make_device(spec, dev)
+    K, V, Q, cu, dS = data["K"], data["V"], data["Q"], data["cu_seqlens"], data["dsketch"]
+    B = int(lens.size)
+    N, H, d = K.shape
+    P = Q.shape[1]
+    tokens = int(lens.sum())
+    sketch = torch.empty((B, H, P, d), dtype=torch.float32, device=dev)
+    lse = torch.empty((N, H), dtype=torch.float32, device=dev)
+    dK, dV = torch.empty_like(K), torch.empty_like(V)
+    dQ = torch.empty((H, P, d), dtype=torch.float32, device=dev)
+    ws = torch.empty(binding.sa_workspace_size(B, N, H, P, d, binding.SA_BF16, 1), dtype=torch.uint8, device=dev)
+
+    def step():
+        binding.sa_sketch_fwd(K, V, cu, Q, spec.scale, out=sketch, lse_out=lse, ws=ws)
+        binding.sa_sketch_bwd(K, V, cu, Q, dS, spec.scale, lse=lse, outs=(dK, dV, dQ), ws=ws)
+
+    for _ in range(args.warmup):
+        step()
+    if binding.sa_get_device_error(ws) != 0:
+        raise RuntimeError("device-side error during warm-up")
+
+    # fwd-only timing (same inputs), for the forward half of the metric
+    stream = torch.cuda.current_stream(dev)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(max(1, args.steps)):
+        binding.sa_sketch_fwd(K, V, cu, Q, spec.scale, out=sketch, lse_out=lse, ws=ws)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    fwd_ms = e0.elapsed_time(e1) / max(1, args.steps)
+
+    # timed region: K steps, barrier + synchronize on both sides, kernel events on
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    binding.sa_timing_enable(True)
+    n_launch0 = binding.sa_launch_count()
+    with Clocks(local) as clk:
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+    launches = binding.sa_launch_count() - n_launch0
+    ms = e0.elapsed_time(e1)
+    fwd_k_ms, fwd_k_n = binding.sa_timing_read(binding.SA_KERNEL_FWD_MAIN)
+    bwd_k_ms, bwd_k_n = binding.sa_timing_read(binding.SA_KERNEL_BWD_MAIN)
+    binding.sa_timing_enable(False)
+    if binding.sa_get_device_error(ws) != 0:
+        raise RuntimeError("device-side error in the timed region")
+    t_max = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
+    ms = float(t_max.item())
+    ms_per_step = ms / args.steps
+    value = tokens * world * args.steps / (ms / 1e3)
+
+    # roofline of the dominant kernel (the backward main kernel) and of the forward
+    eb = 2
+    fw = rf.fwd_work(tokens, B, H, P, d, eb, lse=True)
+    bw = rf.bwd_work(tokens, B, H, P, d, eb, lse_in=True)
+    peak_t = pk["bf16_tflops_sustained"]
+
+    def roof(work, kms, kn, name):
+        if kn == 0:
+            return None
+        avg_s = kms / kn / 1e3
+        t_tensor = work.flops / (peak_t * 1e12)
+        t_hbm = work.bytes / (pk["hbm_gbs"] * 1e9)
+        if t_tensor >= t_hbm:
+            ach, peak, unit, bound = work.flops / avg_s / 1e12, peak_t, "TFLOP/s", "tensor"
+        else:
+            ach, peak, unit, bound = work.bytes / avg_s / 1e9, pk["hbm_gbs"], "GB/s", "hbm"
+        return {"kernel": name, "bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
+                "traffic": traffic_for(name), "avg_launch_ms": kms / kn, "launches": kn,
+                "peak_source": f"{pk['source']} ({'bf16 sustained' if unit == 'TFLOP/s' else 'HBM copy'})",
+                "algorithmic_per_launch": work.flops if unit == "TFLOP/s" else work.bytes}
+
+    bwd_name = binding.sa_main_kernel_name(P, d, binding.SA_BF16, True)
+    fwd_name = binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
+    r_bwd = roof(bw, bwd_k_ms, bwd_k_n, bwd_name)
+    r_fwd = roof(fw, fwd_k_ms, fwd_k_n, fwd_name)
+    step_w = rf.step_work(tokens, B, H, P, d, eb)
+    t_roof = rf.roofline_time(step_w, peak_t, pk["hbm_gbs"])
+
+    e2e = e2e_run(args, spec, dev) if rank == 0 else None
+    cpu = oracle_sample(spec, budget_s=15.0) if (rank == 0 and world == 1) else None
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": workload_config(spec, lens),
+                "fwd": {"value": tokens * world / (fwd_ms / 1e3), "unit": "tokens/s", "ms_per_call": fwd_ms,
+                        "roofline_frac": (rf.roofline_time(fw, peak_t, pk["hbm_gbs"])["time"] * 1e3) / fwd_ms},
+                "step_roofline": {"bound": t_roof["bound"], "ms": t_roof["time"] * 1e3,
+                                  "frac": t_roof["time"] * 1e3 / ms_per_step},
+                "roofline": r_bwd, "roofline_fwd": r_fwd,
+                "cpu_baseline": cpu, "e2e": e2e, "clocks": clk.summary(), "gpu_launches": int(launches),
+                "kernels": {"fwd": fwd_name, "bwd": bwd_name}}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def traffic_for(kernel_name):
+    """DRAM bytes per launch from the committed ncu summary, if it matches the
+    kernel source that is built now; else None."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    try:
+        d = json.load(open(p))
+    except ValueError:
+        return None
+    ent = d.get(kernel_name)
+    if not ent:
+        return None
+    from paper_2609_08443_gb300 import build
+
+    return ent.get("bytes_per_launch") if ent.get("source_hash") == build.source_hash() else None
+
+
+def e2e_run(args, spec, dev):
+    """Same metric through the public API with host buffers: every step copies
+    the inputs from pinned host memory, runs fwd+bwd, copies all results back."""
+    import torch
+
+    from paper_2609_08443_gb300 import binding
+
+    sub = wl.sub_spec(spec, list(range(E2E_USERS)))
+    lens = wl.lengths(sub)
+    d_in = wl.make_device(sub, dev)
+    h = {k: v.to("cpu").pin_memory() for k, v in d_in.items() if hasattr(v, "pin_memory")}
+    del d_in
+    B, H, P, d = sub.B, sub.H, sub.P, sub.d
+    N = int(lens.sum())
+    out_host = {"sketch": torch.empty((B, H, P, d), dtype=torch.float32).pin_memory(),
+                "dK": torch.empty((N, H, d), dtype=torch.bfloat16).pin_memory(),
+                "dV": torch.empty((N, H, d), dtype=torch.bfloat16).pin_memory(),
+                "dQ": torch.empty((H, P, d), dtype=torch.float32).pin_memory()}
+    ws = torch.empty(binding.sa_workspace_size(B, N, H, P, d, binding.SA_BF16, 1), dtype=torch.uint8, device=dev)
+    h2d = sum(v.numel() * v.element_size() for v in h.values())
+    d2h = sum(v.numel() * v.element_size() for v in out_host.values())
+
+    def step():
+        g = {k: v.to(dev, non_blocking=True) for k, v in h.items()}
+        s, lse = binding.sa_sketch_fwd(g["K"], g["V"], g["cu_seqlens"], g["Q"], sub.scale, want_lse=True, ws=ws)
+        dK, dV, dQ = binding.sa_sketch_bwd(g["K"], g["V"], g["cu_seqlens"], g["Q"], g["dsketch"], sub.scale,
+                                           lse=lse, ws=ws)
+        out_host["sketch"].copy_(s, non_blocking=True)
+        out_host["dK"].copy_(dK, non_blocking=True)
+        out_host["dV"].copy_(dV, non_blocking=True)
+        out_host["dQ"].copy_(dQ, non_blocking=True)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize(dev)
+    n = max(2, min(args.steps, 5))
+    t0 = time.perf_counter()
+    for _ in range(n):
+        step()
+    torch.cuda.synchronize(dev)
+    dt = (time.perf_counter() - t0) / n
+    return {"value": N / dt, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "sample": f"{E2E_USERS} of the 128 users (same shapes), host pinned buffers, wall clock",
+            "ms_per_step": dt * 1e3}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    spec = wl.config(CONFIG_ID)
+    lens = wl.lengths(spec)
+    if args.impl == "reference":
+        run_reference(args, spec, lens)
+    else:
+        run_ours(args, spec, lens)
+
+
+if __name__ == "__main__":
+    main()

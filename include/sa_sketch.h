@@ -1,0 +1,138 @@
+/*
+ * sa_sketch.h -- C ABI of libsa_sketch.so, the GB300 (sm_103a) implementation of
+ * the Sketch Attention (SA) sketching step of SequenceO1.
+ *
+ * The operation (paper Sec. 3.1, equations for the affinity S, the prototype-wise
+ * softmax A and the sketch eq:sa-sketch; App. B steps 1-3), for every user b and
+ * head h, with K_b, V_b the user's rows cu_seqlens[b] .. cu_seqlens[b+1]-1:
+ *
+ *     S[j,i]     = scale * sum_c Q[h,j,c] * K_b[i,h,c]           (P x L_b)
+ *     A[:,i]     = softmax over the P prototypes of S[:,i]       (each token
+ *                  spreads unit mass over the prototypes)
+ *     sketch[b,h]= A V_b                                         (P x d)
+ *
+ * No further normalisation is applied (the sketch is the plain weighted sum over
+ * the user's tokens, Sec. 3.1).  Heads are independent copies of the paper's
+ * single-head SA.  The backward is the chain rule of these three steps; the
+ * prototypes are shared by all users (Sec. 3.1), so dQ sums over the batch.
+ * FlashSA (Sec. 4.4) motivates the streaming design: S and A never reach HBM.
+ *
+ * Conventions shared by every entry point
+ *   - All tensors are contiguous, row-major, in device memory, owned by the
+ *     caller.  The library never allocates device memory and keeps no state
+ *     besides per-device caches (kernel attributes, SM count, timing events).
+ *   - K, V, Q, dK, dV all have element type `dt`.  sketch, dsketch, dQ and lse
+ *     are float32.  Element offsets are 64-bit.
+ *   - K, V   : [N, H, d]   packed rows of all users, N = cu_seqlens[B]
+ *     Q      : [H, P, d]   prototypes
+ *     cu     : [B + 1]     int32, cu[0] = 0, non-decreasing, cu[B] = N
+ *     sketch : [B, H, P, d]      lse : [N, H]      dQ : [H, P, d]
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Every call only enqueues work on it and returns; nothing
+ *     synchronises the host.
+ *   - Outputs are overwritten, never accumulated into.  A user with L_b = 0 gets
+ *     an all-zero sketch and contributes nothing to dQ.
+ *   - Inputs and outputs must not overlap.
+ *   - Results are bitwise reproducible for the same inputs, device and
+ *     arguments: every reduction runs in a fixed order (no float atomics).
+ *   - Errors the host can see (NULL pointers, sizes, unsupported shapes, a small
+ *     workspace) are returned synchronously before anything is enqueued.
+ *     Errors only the device can see (bad cu_seqlens contents, a pipeline wait
+ *     that gave up) are written to an error word inside the workspace; the
+ *     kernels of that call then skip their work, and sa_get_device_error()
+ *     reports the code.
+ *   - Not thread-safe for concurrent calls that share one workspace.
+ */
+#ifndef SA_SKETCH_H
+#define SA_SKETCH_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SA_OK = 0,
+  SA_ERR_INVALID_ARG = 1,  /* NULL pointer, negative size, scale not finite     */
+  SA_ERR_UNSUPPORTED = 2,  /* shape or dtype outside what the kernels support   */
+  SA_ERR_WORKSPACE = 3,    /* ws_bytes smaller than sa_workspace_size()          */
+  SA_ERR_CUDA = 4,         /* a CUDA runtime call failed (launch, event, ...)    */
+  SA_ERR_TIMEOUT = 5,      /* a device pipeline wait gave up (device-detected)   */
+  SA_ERR_BAD_SEQLENS = 6   /* cu_seqlens not 0..N non-decreasing (device-detected) */
+} sa_status;
+
+typedef enum { SA_F32 = 0, SA_BF16 = 1 } sa_dtype;
+
+/* Bytes of scratch the caller must pass as `workspace` (device memory, 256-byte
+ * aligned) for a call with these sizes on the current device; `bwd` != 0 sizes
+ * it for sa_sketch_bwd, which needs more.  Returns 0 for invalid sizes.
+ * Supported: 1 <= P <= 1024, 1 <= d <= 128 (d a multiple of 8 for bf16, of 4 for
+ * f32), 1 <= H <= 64, B >= 1, 0 <= N < 2^31. */
+size_t sa_workspace_size(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd);
+
+/* Forward: sketch[b,h] = softmax_proto(scale * Q[h] K_b[:,h]^T) V_b[:,h]
+ * (Sec. 3.1).  `lse` may be NULL; when given it receives, per token and head,
+ * log sum_j exp(S[j,i]) (the softmax statistic FlashSA keeps, Sec. 4.4) so the
+ * backward can skip recomputing it.  `scale` is normally 1/sqrt(d). */
+sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens, int B,
+                        int64_t N, const void* Q, int H, int P, int d, float scale,
+                        sa_dtype dt, float* sketch, float* lse, void* workspace,
+                        size_t ws_bytes, void* stream);
+
+/* Backward of the forward above for upstream gradient dsketch [B,H,P,d] (fp32):
+ *   dV_i = sum_j A[j,i] G_j,   dS = A o (G V^T - colsum(A o G V^T)),
+ *   dK_i = scale sum_j dS[j,i] Q_j,   dQ[h] = scale sum_b sum_i dS[:,i] K_b[i,h]
+ * (chain rule of Sec. 3.1; the paper prints no backward).  `lse` is the forward's
+ * statistic or NULL (then it is recomputed).  dK, dV have type `dt`; dQ is fp32
+ * and fully overwritten (the sum over all users of the batch). */
+sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens, int B,
+                        int64_t N, const void* Q, int H, int P, int d, float scale,
+                        sa_dtype dt, const float* dsketch, const float* lse, void* dK,
+                        void* dV, float* dQ, void* workspace, size_t ws_bytes,
+                        void* stream);
+
+/* Synchronises `stream` and returns the device-detected status of the last call
+ * that used this workspace (SA_OK, SA_ERR_BAD_SEQLENS or SA_ERR_TIMEOUT), or
+ * SA_ERR_CUDA if the stream itself reports an error. */
+sa_status sa_get_device_error(const void* workspace, void* stream);
+
+/* Static English description of a status code. */
+const char* sa_status_string(sa_status s);
+
+/* ---- measurement hooks (used by bench.py; not needed for normal use) ------- */
+
+/* Kernel classes whose launches can be timed with CUDA events. */
+typedef enum { SA_KERNEL_FWD_MAIN = 0, SA_KERNEL_BWD_MAIN = 1, SA_KERNEL_AUX = 2 } sa_kernel_class;
+
+/* Turn event timing of the main kernels on (1) or off (0) and clear the record.
+ * When on, every main-kernel launch is bracketed by CUDA events recorded on the
+ * launching stream (at most 4096 launches are recorded). */
+sa_status sa_timing_enable(int on);
+
+/* Synchronises the recorded events and returns, for kernel class `k`, the sum of
+ * launch durations in milliseconds and the number of launches recorded. */
+sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches);
+
+/* Number of kernels this library has launched in this process. */
+uint64_t sa_launch_count(void);
+
+/* Name of the kernel that a forward (bwd = 0) or backward (bwd = 1) call with
+ * these shapes would use as its main kernel ("tc..." = tcgen05 tensor cores,
+ * "simt..." = CUDA cores).  Static string. */
+const char* sa_main_kernel_name(int P, int d, sa_dtype dt, int bwd);
+
+/* ---- host-side planning (pure C, no GPU; exported for tests) -------------- */
+
+/* The tiling every call applies: user b contributes ceil(L_b / tile) tiles per
+ * head, tiles are ordered (head, user, tile), and worker w of n_workers owns
+ * the contiguous tile range [begin[w], begin[w+1]).  Fills begin[0..n_workers]
+ * from host cu_seqlens; returns SA_ERR_BAD_SEQLENS for invalid offsets. */
+sa_status sa_plan_host(const int32_t* cu_seqlens_host, int B, int H, int tile, int n_workers,
+                       int64_t* begin);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SA_SKETCH_H */

@@ -1,0 +1,238 @@
+"""ctypes binding of libsa_sketch.so (argument marshalling only).
+
+Every function here has the name of the C entry point it calls (see
+``include/sa_sketch.h``).  Torch supplies device memory and the current CUDA
+stream; all arithmetic runs in the library's kernels.  If the library is not
+built or cannot be loaded, every call raises: there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+from typing import Optional, Tuple
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libsa_sketch.so")
+
+SA_F32, SA_BF16 = 0, 1
+SA_KERNEL_FWD_MAIN, SA_KERNEL_BWD_MAIN, SA_KERNEL_AUX = 0, 1, 2
+STATUS = {0: "SA_OK", 1: "SA_ERR_INVALID_ARG", 2: "SA_ERR_UNSUPPORTED", 3: "SA_ERR_WORKSPACE",
+          4: "SA_ERR_CUDA", 5: "SA_ERR_TIMEOUT", 6: "SA_ERR_BAD_SEQLENS"}
+
+_lib = None
+
+
+class SketchError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS.get(status, status)} ({sa_status_string(status)})")
+
+
+def load() -> ctypes.CDLL:
+    """Load the CUDA library (raises if it is missing: no fallback exists)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is not built; run `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64, f32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+    lib.sa_workspace_size.argtypes = [i32, i64, i32, i32, i32, i32, i32]
+    lib.sa_workspace_size.restype = sz
+    lib.sa_sketch_fwd.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp, sz, vp]
+    lib.sa_sketch_fwd.restype = i32
+    lib.sa_sketch_bwd.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp, vp, vp, vp,
+                                  sz, vp]
+    lib.sa_sketch_bwd.restype = i32
+    lib.sa_get_device_error.argtypes = [vp, vp]
+    lib.sa_get_device_error.restype = i32
+    lib.sa_status_string.argtypes = [i32]
+    lib.sa_status_string.restype = ctypes.c_char_p
+    lib.sa_timing_enable.argtypes = [i32]
+    lib.sa_timing_enable.restype = i32
+    lib.sa_timing_read.argtypes = [i32, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64)]
+    lib.sa_timing_read.restype = i32
+    lib.sa_launch_count.argtypes = []
+    lib.sa_launch_count.restype = ctypes.c_uint64
+    lib.sa_main_kernel_name.argtypes = [i32, i32, i32, i32]
+    lib.sa_main_kernel_name.restype = ctypes.c_char_p
+    lib.sa_plan_host.argtypes = [vp, i32, i32, i32, i32, vp]
+    lib.sa_plan_host.restype = i32
+    _lib = lib
+    return lib
+
+
+def _dt(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return SA_BF16
+    if t.dtype == torch.float32:
+        return SA_F32
+    raise TypeError(f"unsupported dtype {t.dtype} (bf16 or fp32)")
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(device) -> ctypes.c_void_p:
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _check(st: int, where: str):
+    if st != 0:
+        raise SketchError(st, where)
+
+
+def _validate(K, V, cu, Q):
+    for name, t in (("K", K), ("V", V), ("Q", Q), ("cu_seqlens", cu)):
+        if not t.is_cuda:
+            raise ValueError(f"{name} must be a CUDA tensor")
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+    if K.dim() != 3 or V.shape != K.shape or Q.dim() != 3 or Q.shape[0] != K.shape[1] or Q.shape[2] != K.shape[2]:
+        raise ValueError(f"shapes K{tuple(K.shape)} V{tuple(V.shape)} Q{tuple(Q.shape)}: want K,V [N,H,d], Q [H,P,d]")
+    if K.dtype != V.dtype or K.dtype != Q.dtype:
+        raise ValueError("K, V and Q must share one dtype")
+    if cu.dtype != torch.int32 or cu.dim() != 1 or cu.numel() < 2:
+        raise ValueError("cu_seqlens must be int32 [B+1]")
+
+
+# ------------------------------------------------------------- C entry points
+
+def sa_workspace_size(B: int, N: int, H: int, P: int, d: int, dt: int, bwd: bool) -> int:
+    return int(load().sa_workspace_size(B, N, H, P, d, dt, int(bool(bwd))))
+
+
+def sa_status_string(status: int) -> str:
+    return load().sa_status_string(status).decode()
+
+
+def sa_main_kernel_name(P: int, d: int, dt: int, bwd: bool) -> str:
+    return load().sa_main_kernel_name(P, d, dt, int(bool(bwd))).decode()
+
+
+def sa_launch_count() -> int:
+    return int(load().sa_launch_count())
+
+
+def sa_timing_enable(on: bool) -> None:
+    _check(load().sa_timing_enable(int(bool(on))), "sa_timing_enable")
+
+
+def sa_timing_read(kernel_class: int) -> Tuple[float, int]:
+    ms, n = ctypes.c_double(), ctypes.c_int64()
+    _check(load().sa_timing_read(kernel_class, ctypes.byref(ms), ctypes.byref(n)), "sa_timing_read")
+    return ms.value, n.value
+
+
+def sa_get_device_error(workspace: torch.Tensor) -> int:
+    return int(load().sa_get_device_error(_ptr(workspace), _stream(workspace.device)))
+
+
+_ws_cache = {}
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    """A cached uint8 device buffer of at least ``nbytes`` (allocated by torch)."""
+    dev = torch.device(device)
+    key = (dev.type, dev.index if dev.index is not None else torch.cuda.current_device())
+    buf = _ws_cache.get(key)
+    if buf is None or buf.numel() < nbytes:
+        buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=dev)
+        _ws_cache[key] = buf
+    return buf
+
+
+def sa_sketch_fwd(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
+                  scale: Optional[float] = None, want_lse: bool = False,
+                  out: Optional[torch.Tensor] = None, lse_out: Optional[torch.Tensor] = None,
+                  ws: Optional[torch.Tensor] = None):
+    """sketch [B,H,P,d] fp32 (and lse [N,H] fp32 when ``want_lse``)."""
+    lib = load()
+    _validate(K, V, cu_seqlens, Q)
+    N, H, d = K.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    dt = _dt(K)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    sketch = out if out is not None else torch.empty((B, H, P, d), dtype=torch.float32, device=K.device)
+    lse = lse_out if lse_out is not None else (
+        torch.empty((N, H), dtype=torch.float32, device=K.device) if want_lse else None)
+    need = lib.sa_workspace_size(B, N, H, P, d, dt, 0)
+    if need == 0:
+        raise SketchError(2, "sa_workspace_size")
+    w = ws if ws is not None else workspace(need, K.device)
+    st = lib.sa_sketch_fwd(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
+                           _ptr(sketch), _ptr(lse), _ptr(w), w.numel(), _stream(K.device))
+    _check(st, "sa_sketch_fwd")
+    return (sketch, lse) if want_lse or lse_out is not None else sketch
+
+
+def sa_sketch_bwd(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
+                  dsketch: torch.Tensor, scale: Optional[float] = None,
+                  lse: Optional[torch.Tensor] = None, outs=None, ws: Optional[torch.Tensor] = None):
+    """(dK, dV, dQ): dK, dV like K; dQ [H,P,d] fp32."""
+    lib = load()
+    _validate(K, V, cu_seqlens, Q)
+    N, H, d = K.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    if dsketch.shape != (B, H, P, d) or dsketch.dtype != torch.float32 or not dsketch.is_contiguous():
+        raise ValueError("dsketch must be contiguous fp32 [B,H,P,d]")
+    if lse is not None and (lse.shape != (N, H) or lse.dtype != torch.float32 or not lse.is_contiguous()):
+        raise ValueError("lse must be contiguous fp32 [N,H]")
+    dt = _dt(K)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    if outs is None:
+        dK, dV = torch.empty_like(K), torch.empty_like(V)
+        dQ = torch.empty((H, P, d), dtype=torch.float32, device=K.device)
+    else:
+        dK, dV, dQ = outs
+    need = lib.sa_workspace_size(B, N, H, P, d, dt, 1)
+    if need == 0:
+        raise SketchError(2, "sa_workspace_size")
+    w = ws if ws is not None else workspace(need, K.device)
+    st = lib.sa_sketch_bwd(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
+                           _ptr(dsketch), _ptr(lse), _ptr(dK), _ptr(dV), _ptr(dQ), _ptr(w), w.numel(),
+                           _stream(K.device))
+    _check(st, "sa_sketch_bwd")
+    return dK, dV, dQ
+
+
+def sa_plan_host(cu_seqlens_host, H: int, tile: int, n_workers: int):
+    """Host copy of the tiling every call applies (pure C; no GPU)."""
+    import numpy as np
+
+    cu = np.ascontiguousarray(cu_seqlens_host, dtype=np.int32)
+    begin = np.zeros(n_workers + 1, dtype=np.int64)
+    st = load().sa_plan_host(cu.ctypes.data, cu.size - 1, H, tile, n_workers, begin.ctypes.data)
+    _check(st, "sa_plan_host")
+    return begin
+
+
+# ------------------------------------------------------------------ autograd
+
+class SketchAttention(torch.autograd.Function):
+    """sketch = softmax_proto(scale Q K^T) V per user and head (Sec. 3.1)."""
+
+    @staticmethod
+    def forward(ctx, K, V, cu_seqlens, Q, scale):
+        sketch, lse = sa_sketch_fwd(K, V, cu_seqlens, Q, scale, want_lse=True)
+        ctx.save_for_backward(K, V, cu_seqlens, Q, lse)
+        ctx.scale = scale
+        return sketch
+
+    @staticmethod
+    def backward(ctx, dsketch):
+        K, V, cu, Q, lse = ctx.saved_tensors
+        dK, dV, dQ = sa_sketch_bwd(K, V, cu, Q, dsketch.contiguous(), ctx.scale, lse=lse)
+        return dK, dV, None, dQ.to(Q.dtype), None
+
+
+def sa_sketch(K, V, cu_seqlens, Q, scale: Optional[float] = None):
+    """Differentiable sketch [B,H,P,d] (fp32) of packed ragged histories."""
+    scale = 1.0 / math.sqrt(K.shape[-1]) if scale is None else float(scale)
+    return SketchAttention.apply(K, V, cu_seqlens, Q, scale)

@@ -1,0 +1,285 @@
+// Host side of libsa_sketch: argument checks, workspace sizing, the choice of
+// kernels for a shape, launches on the caller's stream and the measurement
+// hooks.  Declarations and the meaning of every argument: include/sa_sketch.h.
+#include <atomic>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "sa_kernels.cuh"
+#include "sa_tc.cuh"
+
+namespace {
+
+std::atomic<uint64_t> g_launches{0};
+
+int device_sms() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cache[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    cache[dev] = n;
+  }
+  return cache[dev];
+}
+
+// ------------------------------------------------------------------ timing
+struct TimingRec {
+  cudaEvent_t a = nullptr, b = nullptr;
+  int cls = 0;
+  bool used = false;
+};
+std::mutex g_tmu;
+bool g_timing = false;
+std::vector<TimingRec> g_recs;
+size_t g_nrec = 0;
+constexpr size_t kMaxRecords = 4096;
+
+TimingRec* timing_begin(int cls, cudaStream_t st) {
+  std::lock_guard<std::mutex> lk(g_tmu);
+  if (!g_timing || g_nrec >= kMaxRecords) return nullptr;
+  if (g_recs.size() <= g_nrec) {
+    TimingRec r;
+    if (cudaEventCreate(&r.a) != cudaSuccess || cudaEventCreate(&r.b) != cudaSuccess) return nullptr;
+    g_recs.push_back(r);
+  }
+  TimingRec* r = &g_recs[g_nrec++];
+  r->cls = cls;
+  r->used = cudaEventRecord(r->a, st) == cudaSuccess;
+  return r;
+}
+
+void timing_end(TimingRec* r, cudaStream_t st) {
+  if (r && r->used) r->used = cudaEventRecord(r->b, st) == cudaSuccess;
+}
+
+template <class F>
+sa_status launch(int cls, cudaStream_t st, F&& f) {
+  TimingRec* rec = (cls == SA_KERNEL_AUX) ? nullptr : timing_begin(cls, st);
+  const cudaError_t e = f();
+  g_launches.fetch_add(1, std::memory_order_relaxed);
+  timing_end(rec, st);
+  return e == cudaSuccess ? SA_OK : SA_ERR_CUDA;
+}
+
+#define SA_TRY(x)                      \
+  do {                                 \
+    const sa_status s_ = (x);          \
+    if (s_ != SA_OK) return s_;        \
+  } while (0)
+
+// ------------------------------------------------------------------ planning
+enum class Path { Simt, TcFwd, TcBwd };
+
+struct Plan {
+  Path fwd_path, bwd_path;
+  int T_fwd, W_fwd, T_bwd, W_bwd;
+  sa::WsLayout lay;
+};
+
+bool shape_ok(int B, int64_t N, int H, int P, int d, sa_dtype dt) {
+  if (B < 1 || N < 0 || N >= (int64_t(1) << 31) || H < 1 || H > sa::kMaxH) return false;
+  if (P < 1 || P > sa::kMaxP || d < 1 || d > sa::kMaxD) return false;
+  if (dt != SA_F32 && dt != SA_BF16) return false;
+  return d % (dt == SA_BF16 ? 8 : 4) == 0;
+}
+
+Plan make_plan(int B, int64_t N, int H, int P, int d, sa_dtype dt, bool bwd) {
+  Plan p{};
+  const int sms = device_sms() > 0 ? device_sms() : 1;
+  p.fwd_path = sa::tc_fwd_supported(P, d, dt) ? Path::TcFwd : Path::Simt;
+  p.bwd_path = sa::tc_bwd_supported(P, d, dt) ? Path::TcBwd : Path::Simt;
+  if (p.fwd_path == Path::TcFwd) {
+    p.T_fwd = sa::tc_tile_tokens();
+    p.W_fwd = sa::tc_fwd_workers(sms, P, d);
+  } else {
+    p.T_fwd = sa::simt_tile_tokens();
+    p.W_fwd = sa::simt_workers(sms, P);
+  }
+  if (p.bwd_path == Path::TcBwd) {
+    p.T_bwd = sa::tc_tile_tokens();
+    p.W_bwd = sa::tc_bwd_workers(sms, P, d);
+  } else {
+    p.T_bwd = sa::simt_tile_tokens();
+    p.W_bwd = sa::simt_workers(sms, P);
+  }
+  const int W = (bwd && p.W_bwd > p.W_fwd) ? p.W_bwd : p.W_fwd;
+  p.lay = sa::ws_layout(B, N, H, P, d, W, bwd);
+  return p;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+sa_status check_common(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q,
+                       int H, int P, int d, float scale, sa_dtype dt, const void* ws, size_t ws_bytes,
+                       bool bwd, Plan* plan) {
+  if (!cu || !Q || !ws) return SA_ERR_INVALID_ARG;
+  if (N > 0 && (!K || !V)) return SA_ERR_INVALID_ARG;
+  if (!std::isfinite(scale)) return SA_ERR_INVALID_ARG;
+  if (B < 1 || N < 0 || H < 1 || P < 1 || d < 1) return SA_ERR_INVALID_ARG;
+  if (!shape_ok(B, N, H, P, d, dt)) return SA_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return SA_ERR_INVALID_ARG;
+  if ((K && !aligned16(K)) || (V && !aligned16(V)) || !aligned16(Q)) return SA_ERR_INVALID_ARG;
+  *plan = make_plan(B, N, H, P, d, dt, bwd);
+  if (ws_bytes < plan->lay.total) return SA_ERR_WORKSPACE;
+  return SA_OK;
+}
+
+sa::Args make_args(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q, int H,
+                   int P, int d, float scale, sa_dtype dt, void* ws, const sa::WsLayout& L) {
+  sa::Args a{};
+  char* base = static_cast<char*>(ws);
+  a.K = K;
+  a.V = V;
+  a.Q = Q;
+  a.cu = cu;
+  a.B = B;
+  a.N = N;
+  a.H = H;
+  a.P = P;
+  a.d = d;
+  a.scale = scale;
+  a.dt = dt;
+  a.ws = ws;
+  a.prefix = reinterpret_cast<int64_t*>(base + L.tile_prefix);
+  a.partial = reinterpret_cast<float*>(base + L.partial);
+  a.dq_partial = reinterpret_cast<float*>(base + L.dq_partial);
+  return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t sa_workspace_size(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd) {
+  if (!shape_ok(B, N, H, P, d, dt)) return 0;
+  return make_plan(B, N, H, P, d, dt, bwd != 0).lay.total;
+}
+
+sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                        const void* Q, int H, int P, int d, float scale, sa_dtype dt, float* sketch,
+                        float* lse, void* workspace, size_t ws_bytes, void* stream) {
+  if (!sketch) return SA_ERR_INVALID_ARG;
+  Plan plan;
+  SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, false, &plan));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, plan.lay);
+  char* base = static_cast<char*>(workspace);
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, plan.T_fwd, st); }));
+  if (plan.fwd_path == Path::TcFwd) {
+    SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_tc_fwd(a, plan.W_fwd, sketch, lse, st); }));
+  } else {
+    float* l = lse ? lse : reinterpret_cast<float*>(base + plan.lay.lse);
+    SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_simt_lse(a, l, st); }));
+    SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_simt_fwd(a, plan.W_fwd, l, sketch, st); }));
+  }
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_sketch(a, plan.W_fwd, sketch, st); }));
+  return SA_OK;
+}
+
+sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                        const void* Q, int H, int P, int d, float scale, sa_dtype dt, const float* dsketch,
+                        const float* lse, void* dK, void* dV, float* dQ, void* workspace, size_t ws_bytes,
+                        void* stream) {
+  if (!dsketch || !dQ || (N > 0 && (!dK || !dV))) return SA_ERR_INVALID_ARG;
+  Plan plan;
+  SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, true, &plan));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, plan.lay);
+  char* base = static_cast<char*>(workspace);
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, plan.T_bwd, st); }));
+  const float* l = lse;
+  if (!l) {
+    float* scratch = reinterpret_cast<float*>(base + plan.lay.lse);
+    if (plan.bwd_path == Path::TcBwd) {
+      SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tc_lse(a, scratch, st); }));
+    } else {
+      SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_simt_lse(a, scratch, st); }));
+    }
+    l = scratch;
+  }
+  if (plan.bwd_path == Path::TcBwd) {
+    SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
+                  [&] { return sa::launch_tc_bwd(a, plan.W_bwd, dsketch, l, dK, dV, st); }));
+  } else {
+    float* Dco = reinterpret_cast<float*>(base + plan.lay.dcoef);
+    SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
+                  [&] { return sa::launch_simt_bwd_tokens(a, dsketch, l, dK, dV, Dco, st); }));
+    SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_simt_bwd_dq(a, plan.W_bwd, dsketch, l, Dco, st); }));
+  }
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, plan.W_bwd, dQ, st); }));
+  return SA_OK;
+}
+
+sa_status sa_get_device_error(const void* workspace, void* stream) {
+  if (!workspace) return SA_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return SA_ERR_CUDA;
+  uint32_t err = 0;
+  if (cudaMemcpy(&err, workspace, sizeof(err), cudaMemcpyDeviceToHost) != cudaSuccess) return SA_ERR_CUDA;
+  return static_cast<sa_status>(err);
+}
+
+const char* sa_status_string(sa_status s) {
+  switch (s) {
+    case SA_OK: return "ok";
+    case SA_ERR_INVALID_ARG: return "invalid argument (null pointer, misaligned buffer or bad size)";
+    case SA_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+    case SA_ERR_WORKSPACE: return "workspace smaller than sa_workspace_size()";
+    case SA_ERR_CUDA: return "CUDA runtime error";
+    case SA_ERR_TIMEOUT: return "a device pipeline wait gave up (bounded wait expired)";
+    case SA_ERR_BAD_SEQLENS: return "cu_seqlens is not 0..N non-decreasing";
+  }
+  return "unknown status";
+}
+
+sa_status sa_timing_enable(int on) {
+  std::lock_guard<std::mutex> lk(g_tmu);
+  g_timing = on != 0;
+  g_nrec = 0;
+  return SA_OK;
+}
+
+sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches) {
+  if (!total_ms || !launches) return SA_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_tmu);
+  double tot = 0.0;
+  int64_t n = 0;
+  for (size_t i = 0; i < g_nrec; ++i) {
+    TimingRec& r = g_recs[i];
+    if (r.cls != int(k) || !r.used) continue;
+    if (cudaEventSynchronize(r.b) != cudaSuccess) return SA_ERR_CUDA;
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) return SA_ERR_CUDA;
+    tot += ms;
+    ++n;
+  }
+  *total_ms = tot;
+  *launches = n;
+  return SA_OK;
+}
+
+uint64_t sa_launch_count(void) { return g_launches.load(); }
+
+const char* sa_main_kernel_name(int P, int d, sa_dtype dt, int bwd) {
+  if (bwd) return sa::tc_bwd_supported(P, d, dt) ? sa::tc_bwd_name(P, d) : "simt_bwd_tokens_kernel";
+  return sa::tc_fwd_supported(P, d, dt) ? sa::tc_fwd_name(P, d) : "simt_fwd_agg_kernel";
+}
+
+sa_status sa_plan_host(const int32_t* cu, int B, int H, int tile, int n_workers, int64_t* begin) {
+  if (!cu || !begin || B < 1 || H < 1 || tile < 1 || n_workers < 1) return SA_ERR_INVALID_ARG;
+  if (cu[0] != 0) return SA_ERR_BAD_SEQLENS;
+  int64_t tph = 0;
+  for (int b = 0; b < B; ++b) {
+    const int64_t L = int64_t(cu[b + 1]) - int64_t(cu[b]);
+    if (L < 0) return SA_ERR_BAD_SEQLENS;
+    tph += (L + tile - 1) / tile;
+  }
+  const int64_t total = tph * H;
+  for (int w = 0; w <= n_workers; ++w) begin[w] = sa::range_begin(total, n_workers, w);
+  return SA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,39 @@
+// Internal interface between the host API (sa_api.cu) and the kernel files.
+#pragma once
+#include "sa_common.cuh"
+
+namespace sa {
+
+// Everything a kernel needs about one call (passed by value as a kernel arg).
+struct Args {
+  const void* K;
+  const void* V;
+  const void* Q;
+  const int32_t* cu;
+  int B;
+  int64_t N;
+  int H, P, d;
+  float scale;
+  sa_dtype dt;
+  void* ws;            // workspace base (header)
+  int64_t* prefix;     // per-head tile prefix [B + 1]
+  float* partial;      // [W][2][P][d]
+  float* dq_partial;   // [W][H][P][d]
+};
+
+// planner / finalize (sa_simt.cu)
+cudaError_t launch_plan(const Args& a, int T, cudaStream_t st);
+cudaError_t launch_finalize_sketch(const Args& a, int W, float* sketch, cudaStream_t st);
+cudaError_t launch_finalize_dq(const Args& a, int W, float* dQ, cudaStream_t st);
+
+// CUDA-core path (sa_simt.cu)
+int simt_tile_tokens();
+int simt_workers(int num_sms, int P);
+cudaError_t launch_simt_lse(const Args& a, float* lse, cudaStream_t st);
+cudaError_t launch_simt_fwd(const Args& a, int W, const float* lse, float* sketch, cudaStream_t st);
+cudaError_t launch_simt_bwd_tokens(const Args& a, const float* dsk, const float* lse, void* dK, void* dV,
+                                   float* Dco, cudaStream_t st);
+cudaError_t launch_simt_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
+                               cudaStream_t st);
+
+}  // namespace sa

@@ -1,0 +1,19 @@
+// Interface of the tcgen05 / TMEM / TMA kernels (sm_103a).
+#pragma once
+#include "sa_kernels.cuh"
+
+namespace sa {
+
+bool tc_fwd_supported(int P, int d, sa_dtype dt);
+bool tc_bwd_supported(int P, int d, sa_dtype dt);
+const char* tc_fwd_name(int P, int d);
+const char* tc_bwd_name(int P, int d);
+int tc_tile_tokens();
+int tc_fwd_workers(int num_sms, int P, int d);
+int tc_bwd_workers(int num_sms, int P, int d);
+cudaError_t launch_tc_fwd(const Args& a, int W, float* sketch, float* lse, cudaStream_t st);
+cudaError_t launch_tc_lse(const Args& a, float* lse, cudaStream_t st);
+cudaError_t launch_tc_bwd(const Args& a, int W, const float* dsk, const float* lse, void* dK, void* dV,
+                          cudaStream_t st);
+
+}  // namespace sa

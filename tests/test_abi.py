@@ -1,0 +1,98 @@
+"""The C ABI library loads and exports every symbol its header declares;
+host-side argument checks return their codes without touching a GPU."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2609_08443_gb300 import binding, build
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "sa_sketch.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return binding.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(sa_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for must in ("sa_workspace_size", "sa_sketch_fwd", "sa_sketch_bwd", "sa_get_device_error",
+                 "sa_status_string"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), f"{name} declared in sa_sketch.h but not exported"
+
+
+def test_status_strings(lib):
+    for code in range(7):
+        s = binding.sa_status_string(code)
+        assert s and s != "unknown status"
+    assert binding.sa_status_string(99) == "unknown status"
+
+
+def test_workspace_size_rejects_bad_shapes(lib):
+    assert binding.sa_workspace_size(1, 10, 1, 0, 64, 1, 0) == 0       # P = 0
+    assert binding.sa_workspace_size(1, 10, 1, 2048, 64, 1, 0) == 0    # P too large
+    assert binding.sa_workspace_size(1, 10, 1, 64, 12, 1, 0) == 0      # d not multiple of 8 (bf16)
+    assert binding.sa_workspace_size(0, 10, 1, 64, 64, 1, 0) == 0      # B = 0
+    assert binding.sa_workspace_size(1, 2**31, 1, 64, 64, 1, 0) == 0   # N too large
+    a = binding.sa_workspace_size(4, 1000, 2, 256, 64, 1, 0)
+    b = binding.sa_workspace_size(4, 1000, 2, 256, 64, 1, 1)
+    assert a > 0 and b >= a and a % 256 == 0 and b % 256 == 0
+
+
+def _fwd(lib, **kw):
+    args = dict(K=256, V=512, cu=768, B=2, N=100, Q=1024, H=2, P=64, d=64, scale=0.125, dt=1,
+                sketch=2048, lse=None, ws=4096, wsb=1 << 30)
+    args.update(kw)
+    vp = ctypes.c_void_p
+    return lib.sa_sketch_fwd(vp(args["K"]), vp(args["V"]), vp(args["cu"]), args["B"], args["N"], vp(args["Q"]),
+                             args["H"], args["P"], args["d"], args["scale"], args["dt"], vp(args["sketch"]),
+                             vp(args["lse"]) if args["lse"] else None, vp(args["ws"]), args["wsb"], None)
+
+
+def test_host_checks_return_codes_before_any_launch(lib):
+    # fake, never-dereferenced addresses: only the host checks run
+    assert _fwd(lib, sketch=0) == 1                      # NULL output
+    assert _fwd(lib, cu=0) == 1                          # NULL offsets
+    assert _fwd(lib, scale=float("nan")) == 1            # non-finite scale
+    assert _fwd(lib, ws=4096 + 8) == 1                   # workspace not 256-aligned
+    assert _fwd(lib, K=256 + 2) == 1                     # K not 16-byte aligned
+    assert _fwd(lib, P=4096) == 2                        # unsupported P
+    assert _fwd(lib, d=200) == 2                         # unsupported d
+    assert _fwd(lib, dt=7) == 2                          # unknown dtype
+    assert _fwd(lib, wsb=16) == 3                        # workspace too small
+
+
+def test_plan_host_covers_every_tile_once(lib):
+    rng = np.random.default_rng(0)
+    for lens in ([0], [1], [128], [129], [0, 0, 5], list(rng.integers(0, 600, size=4100)),
+                 [100000] * 3 + [0, 1, 127, 128, 129]):
+        cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        for H in (1, 8):
+            for W in (1, 7, 152, 10000):
+                begin = binding.sa_plan_host(cu, H, 128, W)
+                tiles = H * sum((L + 127) // 128 for L in lens)
+                assert begin[0] == 0 and begin[-1] == tiles
+                sizes = np.diff(begin)
+                assert np.all(sizes >= 0) and sizes.max() - sizes.min() <= 1
+
+
+def test_plan_host_rejects_bad_offsets(lib):
+    with pytest.raises(binding.SketchError):
+        binding.sa_plan_host(np.array([0, 5, 3], np.int32), 1, 128, 4)
+    with pytest.raises(binding.SketchError):
+        binding.sa_plan_host(np.array([1, 5], np.int32), 1, 128, 4)

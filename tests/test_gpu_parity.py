@@ -1,0 +1,75 @@
+"""CUDA path vs the fp64 oracle, element by element, on seeded inputs.
+
+Sizes span several 128-token tiles with ragged tails, empty users and users
+long enough to be cut across workers.  Tolerance: max|gpu - oracle| <=
+1e-4 max|oracle| for fp32 inputs, 2e-2 max|oracle| for bf16 inputs.
+"""
+import numpy as np
+import pytest
+import torch
+
+import harness
+from paper_2609_08443_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+RAGGED = [0, 1, 127, 128, 129, 300, 0, 1000, 17, 2049]
+
+SHAPES = [
+    # (P, d, dtype, H)
+    (64, 64, wl.F32, 1),
+    (256, 64, wl.BF16, 2),
+    (512, 128, wl.BF16, 2),
+    (256, 128, wl.BF16, 1),
+    (512, 64, wl.BF16, 1),
+    (128, 64, wl.BF16, 3),
+    (96, 32, wl.BF16, 1),
+    (200, 128, wl.F32, 1),
+    (1024, 64, wl.BF16, 1),
+    (1, 8, wl.BF16, 1),
+]
+
+
+@pytest.mark.parametrize("P,d,dt,H", SHAPES, ids=lambda x: str(x))
+def test_ragged_fwd_bwd(cuda_lib, P, d, dt, H):
+    spec = wl.custom(RAGGED, H=H, P=P, d=d, dtype=dt, seed=P + d)
+    harness.check_spec(spec, bwd=True)
+
+
+@pytest.mark.parametrize("pass_lse", [True, False])
+def test_bwd_with_and_without_saved_lse(cuda_lib, pass_lse):
+    spec = wl.custom([513, 77, 0, 1300], H=2, P=256, d=64, dtype=wl.BF16, seed=5)
+    harness.check_spec(spec, bwd=True, pass_lse=pass_lse)
+
+
+def test_config1_full(cuda_lib):
+    """Single user, L=4096, H=1, d=64, P=64, fp32, forward (full size)."""
+    harness.check_spec(wl.config(1), bwd=False)
+
+
+def test_config2_full(cuda_lib):
+    """32 users U[1024,16384], H=4, d=64, P=256, bf16, forward (full size)."""
+    harness.check_spec(wl.config(2), bwd=False)
+
+
+def test_config3_subbatch(cuda_lib):
+    """Training-step shape of config 3 on 6 of its users (full lengths)."""
+    spec = wl.config(3)
+    lens = wl.lengths(spec)
+    users = [int(np.argmax(lens)), int(np.argmin(lens)), 0, 1, 2, 3]
+    harness.check_spec(wl.sub_spec(spec, users), bwd=True)
+
+
+def test_config4_subbatch(cuda_lib):
+    """100K-token users, H=8, d=128, P=512, Q ~ N(0, 0.02): 2 users."""
+    spec = wl.sub_spec(wl.config(4), [0, 1])
+    harness.check_spec(spec, bwd=True)
+
+
+def test_config5_subbatch(cuda_lib):
+    """One 1M-token user mixed with 40 short users of config 5."""
+    spec = wl.config(5)
+    lens = wl.lengths(spec)
+    long_u = int(np.nonzero(lens == 1048576)[0][0])
+    short_u = [int(u) for u in np.nonzero(lens < 1048576)[0][:40]]
+    harness.check_spec(wl.sub_spec(spec, [short_u[0], long_u] + short_u[1:]), bwd=True)
