@@ -118,6 +118,12 @@ sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches)
 /* Number of kernels this library has launched in this process. */
 uint64_t sa_launch_count(void);
 
+/* Kernel selection for all later calls in this process: 0 (default) lets each
+ * call pick the tensor-core kernels where its shape is supported, 1 forces the
+ * CUDA-core kernels everywhere (a cross-check of the two).  The workspace size
+ * depends on the selection: size it after choosing. */
+sa_status sa_select_path(int path);
+
 /* Name of the kernel that a forward (bwd = 0) or backward (bwd = 1) call with
  * these shapes would use as its main kernel ("tc..." = tcgen05 tensor cores,
  * "simt..." = CUDA cores).  Static string. */

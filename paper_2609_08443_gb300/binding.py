@@ -59,6 +59,8 @@ def load() -> ctypes.CDLL:
     lib.sa_launch_count.restype = ctypes.c_uint64
     lib.sa_main_kernel_name.argtypes = [i32, i32, i32, i32]
     lib.sa_main_kernel_name.restype = ctypes.c_char_p
+    lib.sa_select_path.argtypes = [i32]
+    lib.sa_select_path.restype = i32
     lib.sa_plan_host.argtypes = [vp, i32, i32, i32, i32, vp]
     lib.sa_plan_host.restype = i32
     _lib = lib
@@ -116,6 +118,11 @@ def sa_main_kernel_name(P: int, d: int, dt: int, bwd: bool) -> str:
 
 def sa_launch_count() -> int:
     return int(load().sa_launch_count())
+
+
+def sa_select_path(path: int) -> None:
+    """0: tensor-core kernels where supported (default); 1: CUDA cores only."""
+    _check(load().sa_select_path(int(path)), "sa_select_path")
 
 
 def sa_timing_enable(on: bool) -> None:

@@ -7,10 +7,15 @@
 #include <mutex>
 #include <vector>
 
+#include <cuda.h>
+
 #include "sa_kernels.cuh"
 #include "sa_tc.cuh"
+#include "sa_tc_common.cuh"
 
 namespace {
+
+std::atomic<int> g_path{0};  // 0 = choose per shape, 1 = CUDA cores only
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -147,10 +152,77 @@ sa::Args make_args(const void* K, const void* V, const int32_t* cu, int B, int64
   a.prefix = reinterpret_cast<int64_t*>(base + L.tile_prefix);
   a.partial = reinterpret_cast<float*>(base + L.partial);
   a.dq_partial = reinterpret_cast<float*>(base + L.dq_partial);
+  a.lse_scratch = reinterpret_cast<float*>(base + L.lse);
   return a;
 }
 
 }  // namespace
+
+// ------------------------------------------------------- tensor-core helpers
+namespace sa {
+
+bool tc_path_enabled() { return g_path.load() == 0; }
+
+namespace tcc {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// K or V [N, H, D] bf16 -> boxes of [128 tokens][1 head][64 features], 128-byte swizzle;
+// rows past N read as zero.
+bool make_kv_map(CUtensorMap* m, const void* base, int64_t N, int H, int D) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || N <= 0) return false;
+  const cuuint64_t dims[3] = {cuuint64_t(D), cuuint64_t(H), cuuint64_t(N)};
+  const cuuint64_t strides[2] = {cuuint64_t(D) * 2, cuuint64_t(H) * D * 2};
+  const cuuint32_t box[3] = {64, 1, 128};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Q [H, P, D] bf16 -> boxes of [box_rows prototypes][64 features] of one head.
+bool make_q_map(CUtensorMap* m, const void* Q, int H, int P, int D, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {cuuint64_t(D), cuuint64_t(P), cuuint64_t(H)};
+  const cuuint64_t strides[2] = {cuuint64_t(D) * 2, cuuint64_t(P) * D * 2};
+  const cuuint32_t box[3] = {64, cuuint32_t(box_rows), 1};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(Q), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool device_is_sm103() {
+  int dev = 0, major = 0, minor = 0, smem = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess) return false;
+  if (cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) return false;
+  if (cudaDeviceGetAttribute(&smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
+  return major == 10 && minor == 3 && smem >= 232448;
+}
+
+int device_sm_count() { return device_sms() > 0 ? device_sms() : 1; }
+
+}  // namespace tcc
+}  // namespace sa
 
 extern "C" {
 
@@ -170,7 +242,12 @@ sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens,
   char* base = static_cast<char*>(workspace);
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, plan.T_fwd, st); }));
   if (plan.fwd_path == Path::TcFwd) {
-    SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_tc_fwd(a, plan.W_fwd, sketch, lse, st); }));
+    float* l = lse;
+    if (sa::tc_fwd_needs_lse_pass_d(P, d)) {
+      if (!l) l = a.lse_scratch;
+      SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tc_lse(a, l, st); }));
+    }
+    SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_tc_fwd(a, plan.W_fwd, sketch, l, st); }));
   } else {
     float* l = lse ? lse : reinterpret_cast<float*>(base + plan.lay.lse);
     SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_simt_lse(a, l, st); }));
@@ -262,6 +339,12 @@ sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches)
 }
 
 uint64_t sa_launch_count(void) { return g_launches.load(); }
+
+sa_status sa_select_path(int path) {
+  if (path != 0 && path != 1) return SA_ERR_INVALID_ARG;
+  g_path.store(path);
+  return SA_OK;
+}
 
 const char* sa_main_kernel_name(int P, int d, sa_dtype dt, int bwd) {
   if (bwd) return sa::tc_bwd_supported(P, d, dt) ? sa::tc_bwd_name(P, d) : "simt_bwd_tokens_kernel";

@@ -19,6 +19,7 @@ struct Args {
   int64_t* prefix;     // per-head tile prefix [B + 1]
   float* partial;      // [W][2][P][d]
   float* dq_partial;   // [W][H][P][d]
+  float* lse_scratch;  // [N][H] workspace copy of lse when the caller passes none
 };
 
 // planner / finalize (sa_simt.cu)

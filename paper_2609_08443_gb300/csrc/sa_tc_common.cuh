@@ -1,0 +1,120 @@
+// Pieces shared by the tensor-core kernels: the tile walker every warp role
+// uses to follow its worker's range, TMA tensor maps, TMEM sizing and the
+// epilogue that stores a sketch block from TMEM.
+#pragma once
+#include <cuda.h>
+
+#include "sa_kernels.cuh"
+#include "sa_ptx.cuh"
+
+namespace sa {
+namespace tcc {
+
+constexpr int T = 128;           // tokens per tile = UMMA M
+constexpr int kThreads = 384;    // 12 warps
+constexpr int kSoftWarp0 = 4;    // warps 4..11: softmax / epilogue
+constexpr int kSoftWarps = 8;
+
+__host__ __device__ constexpr int tmem_cols_for(int c) {
+  return c <= 32 ? 32 : c <= 64 ? 64 : c <= 128 ? 128 : c <= 256 ? 256 : 512;
+}
+
+// Follows worker tiles [tb, te) in (head, user, tile) order; all warp roles
+// construct their own walker and see the same sequence.
+struct TileWalker {
+  const int64_t* prefix;
+  const int32_t* cu;
+  int B, Tt;
+  int64_t tph, t, tb, te;
+  int h, b;
+  int64_t k, nk, tok0, seg0, seg1;
+  int n;
+  bool seg_first, seg_last;
+
+  __device__ TileWalker(const Args& a, int64_t tb_, int64_t te_, int T_)
+      : prefix(a.prefix), cu(a.cu), B(a.B), Tt(T_), t(tb_), tb(tb_), te(te_) {
+    tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
+    if (t < te) relocate();
+  }
+  __device__ void relocate() {
+    const TileRef r = locate_tile(t, tph, prefix, cu, B, Tt);
+    h = r.h;
+    b = r.b;
+    seg0 = r.seg0;
+    seg1 = r.seg1;
+    nk = seg1 - seg0;
+    k = t - seg0;
+    fields();
+  }
+  __device__ void fields() {
+    const int64_t L = int64_t(cu[b + 1]) - int64_t(cu[b]);
+    tok0 = int64_t(cu[b]) + k * Tt;
+    const int64_t left = L - k * Tt;
+    n = int(left < Tt ? left : Tt);
+    seg_first = (k == 0) || (t == tb);
+    seg_last = (k == nk - 1) || (t == te - 1);
+  }
+  __device__ void next() {
+    ++t;
+    if (t >= te) return;
+    if (k + 1 < nk) {
+      ++k;
+      fields();
+    } else {
+      relocate();
+    }
+  }
+};
+
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+  if (ptx::mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = ptx::globaltimer();
+  while (!ptx::mbar_try_wait(bar, parity))
+    if (ptx::globaltimer() - t0 > limit_ns) return false;
+  return true;
+}
+
+// Sketch block (PS prototypes x D) from TMEM to global memory.
+//  TRANS (D = 128): TMEM holds O^T: lane = feature d, column = prototype.
+//  else (D = 64):   TMEM holds O in PS/128 blocks: lane = prototype, column = d.
+template <int D, int PS, bool TRANS, int O_COL>
+__device__ __forceinline__ void store_sketch(uint32_t tmem, uint32_t lane_off, int sw, int q, int lane, float* dst) {
+  float v[32];
+  if (TRANS) {
+    const int d = 32 * q + lane;
+#pragma unroll 1
+    for (int c = 0; c < PS / 2 / 32; ++c) {
+      const int pbase = sw * (PS / 2) + 32 * c;
+      ptx::tmem_ld32(tmem + lane_off + O_COL + pbase, v);
+      ptx::tmem_ld_wait();
+#pragma unroll
+      for (int k = 0; k < 32; ++k) dst[int64_t(pbase + k) * D + d] = v[k];
+    }
+  } else {
+    constexpr int NB = PS / 128;
+    const int blk = NB == 2 ? sw : 0;
+    const int p = 128 * blk + 32 * q + lane;
+    const int c0 = NB == 2 ? 0 : 32 * sw;
+    const int c1 = NB == 2 ? D : c0 + 32;
+#pragma unroll 1
+    for (int c = c0; c < c1; c += 32) {
+      ptx::tmem_ld32(tmem + lane_off + O_COL + blk * D + c, v);
+      ptx::tmem_ld_wait();
+      float4* o = reinterpret_cast<float4*>(dst + int64_t(p) * D + c);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) o[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+    }
+  }
+}
+
+// ------------------------------------------------------------- host helpers
+bool make_kv_map(CUtensorMap* m, const void* base, int64_t N, int H, int D);
+bool make_q_map(CUtensorMap* m, const void* Q, int H, int P, int D, int box_rows);
+bool device_is_sm103();
+int device_sm_count();
+
+}  // namespace tcc
+
+bool tc_path_enabled();
+
+}  // namespace sa

@@ -1,13 +1,660 @@
-// tcgen05 forward kernel (sm_103a).  Not yet enabled: every shape takes the
-// CUDA-core path until this kernel passes its parity tests.
+// tcgen05 / TMEM / TMA forward kernels of the SA sketching step (sm_103a).
+//
+// One CTA per SM walks a contiguous range of 128-token tiles (ragged tiling of
+// sa_common.cuh).  Per tile (paper Sec. 3.1; FlashSA's streaming scheme of
+// Sec. 4.4, S and A never leave the SM):
+//   1. TMA brings the tile's K and V rows ([128 tokens][d] bf16, 128-byte
+//      swizzle) into a ring of shared-memory slots; the prototype block Q
+//      ([PS][d]) stays resident while the head does not change.
+//   2. UMMA  S^T = K Q^T  (M = 128 tokens, N = PS prototypes, K = d) into TMEM,
+//      so each token's P scores lie in one TMEM lane.
+//   3. Eight softmax warps read the scores into registers (one token per
+//      thread, half of the prototypes per warpgroup), normalise over the
+//      prototypes -- either with their own max / sum (fused mode, all P in
+//      this CTA) or with a given per-token log-sum-exp (sliced mode) -- and
+//      write the weights A as bf16 into shared memory.
+//   4. UMMA accumulates the sketch in TMEM:  O = A V  (d = 64: M = prototypes,
+//      N = d) or  O^T = V^T A^T  (d = 128: M = d, N = prototypes).
+//   5. When a user's segment ends the sketch (or a worker's piece of it) is
+//      read back from TMEM and stored.
+// Warp roles: 0 = TMA producer, 1 = UMMA issuer, 2 = TMEM allocator,
+// 4..11 = softmax + epilogue.  Every wait is bounded (sa_ptx.cuh).
+#include <cuda.h>
+
+#include <cstdio>
+
+#include "sa_ptx.cuh"
 #include "sa_tc.cuh"
+#include "sa_tc_common.cuh"
 
 namespace sa {
+namespace tcf {
 
-bool tc_fwd_supported(int, int, sa_dtype) { return false; }
-const char* tc_fwd_name(int, int) { return "tc_fwd"; }
-int tc_tile_tokens() { return 128; }
-int tc_fwd_workers(int num_sms, int, int) { return num_sms; }
-cudaError_t launch_tc_fwd(const Args&, int, float*, float*, cudaStream_t) { return cudaErrorNotSupported; }
+using namespace ptx;
+using namespace tcc;
+
+enum Mode { kFused = 0, kSliced = 1 };
+
+template <int D, int PS, int MODE>
+struct Cfg {
+  static constexpr int KV_TILE = T * D * 2;
+  static constexpr int Q_BYTES = PS * D * 2;
+  static constexpr int W_BYTES = T * PS * 2;
+  static constexpr int NSLOT = (D == 128) ? 3 : 6;
+  static constexpr int STATS = (MODE == kFused) ? 2 * T * 8 : 0;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_RING = OFF_Q + Q_BYTES;
+  static constexpr int OFF_W = OFF_RING + NSLOT * KV_TILE;
+  static constexpr int OFF_STATS = OFF_W + W_BYTES;
+  static constexpr int OFF_BAR = OFF_STATS + STATS;
+  static constexpr int NBAR = 2 * NSLOT + 12;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // tmem address, abort flag
+  static constexpr int SMEM = OFF_MISC + 16;
+  static constexpr bool TRANS = (D == 128);  // O^T = V^T A^T
+  static constexpr int O_COLS = TRANS ? PS : (PS / 128) * D;
+  static constexpr int S_COL = 0;
+  static constexpr int O_COL = PS;
+  static constexpr int TMEM_COLS = tmem_cols_for(PS + O_COLS);
+  static constexpr int HALF = PS / 2;  // prototypes per softmax warpgroup
+};
+
+template <int D, int PS, int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_fwd_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                  const __grid_constant__ CUtensorMap tmQ, Args a, float* __restrict__ sketch,
+                  float* __restrict__ lse_out, const float* __restrict__ lse_in) {
+  using C = Cfg<D, PS, MODE>;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (ws_failed(a.ws)) return;
+  if (smem_u32(smem) & 1023u) {  // 128-byte swizzle atoms need 1024-byte alignment
+    if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xA11u);
+    return;
+  }
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t sQ = sbase + C::OFF_Q, sRing = sbase + C::OFF_RING, sW = sbase + C::OFF_W;
+  const uint32_t bar0 = sbase + C::OFF_BAR;
+  auto ring_full = [&](int s) { return bar0 + 8u * s; };
+  auto ring_empty = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
+  const uint32_t q_full = bar0 + 8u * (2 * C::NSLOT + 0), q_empty = q_full + 8, s_full = q_full + 16,
+                 s_empty = q_full + 24, w_full = q_full + 32, w_empty = q_full + 40, o_full = q_full + 48,
+                 o_empty = q_full + 56, drain = q_full + 64, st_ready = q_full + 72, st_used = q_full + 80;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+
+  const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
+  const int64_t total = tph * a.H;
+  const int W = gridDim.x, wk = blockIdx.x, slice = blockIdx.y;
+  const int p0 = slice * PS;
+  const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
+  const int ntiles = int(te - tb);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(ring_full(s), 1);
+      mbar_init(ring_empty(s), 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    mbar_init(s_full, 1);
+    mbar_init(s_empty, kSoftWarps);
+    mbar_init(w_full, kSoftWarps);
+    mbar_init(w_empty, 1);
+    mbar_init(o_full, 1);
+    mbar_init(o_empty, kSoftWarps);
+    mbar_init(drain, 1);
+    mbar_init(st_ready, kSoftWarps);
+    mbar_init(st_used, kSoftWarps);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (ntiles > 0) {
+    if (warp == 0 && lane == 0) {
+      // ------------------------------------------------------ TMA producer
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      tma_prefetch_desc(&tmQ);
+      TileWalker it(a, tb, te, T), pv(a, tb, te, T);
+      int hc = 0, prev_h = -1;
+      uint32_t e = 0;
+      bool ok = true;
+      for (int li = 0; li <= ntiles && ok; ++li) {
+        if (li < ntiles) {
+          if (it.h != prev_h) {
+            if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0x101);
+            if (!ok) break;
+            mbar_arrive_expect_tx(q_full, C::Q_BYTES);
+#pragma unroll
+            for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.h);
+            prev_h = it.h;
+            ++hc;
+          }
+          const int s = int(e % C::NSLOT);
+          if (e >= uint32_t(C::NSLOT)) ok = mbar_wait(ring_empty(s), ((e / C::NSLOT) + 1) & 1, abort_flag, a.ws, 0x102);
+          if (!ok) break;
+          mbar_arrive_expect_tx(ring_full(s), C::KV_TILE);
+#pragma unroll
+          for (int dh = 0; dh < D / 64; ++dh)
+            tma_load_3d(sRing + s * C::KV_TILE + dh * T * 128, &tmK, ring_full(s), 64 * dh, it.h, int(it.tok0));
+          ++e;
+          it.next();
+        }
+        if (li >= 1) {
+          const int s = int(e % C::NSLOT);
+          if (e >= uint32_t(C::NSLOT)) ok = mbar_wait(ring_empty(s), ((e / C::NSLOT) + 1) & 1, abort_flag, a.ws, 0x103);
+          if (!ok) break;
+          mbar_arrive_expect_tx(ring_full(s), C::KV_TILE);
+#pragma unroll
+          for (int dh = 0; dh < D / 64; ++dh)
+            tma_load_3d(sRing + s * C::KV_TILE + dh * T * 128, &tmV, ring_full(s), 64 * dh, pv.h, int(pv.tok0));
+          ++e;
+          pv.next();
+        }
+      }
+      // drain loads still in flight before the CTA may exit
+      if (!ok) {
+        for (uint32_t k = (e > uint32_t(C::NSLOT) ? e - C::NSLOT : 0); k < e; ++k)
+          mbar_wait_bounded(ring_full(int(k % C::NSLOT)), (k / C::NSLOT) & 1, 200000000ull);
+      }
+    } else if (warp == 1 && lane == 0) {
+      // ------------------------------------------------------ UMMA issuer
+      constexpr uint32_t idS = idesc_bf16(128, PS, 0, 0);
+      constexpr uint32_t idO = C::TRANS ? idesc_bf16(128, PS, 1, 1) : idesc_bf16(128, D, 1, 1);
+      TileWalker cur(a, tb, te, T), nxt(a, tb, te, T);
+      nxt.next();
+      uint32_t e = 0;
+      int hc = 0, sc = 0;
+      bool ok = mbar_wait(q_full, 0, abort_flag, a.ws, 0x201);
+      auto issue_S = [&](uint32_t slot) {
+        const uint32_t kaddr = sRing + slot * C::KV_TILE;
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k) {
+          const uint64_t ad = sdesc(kaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024);
+          const uint64_t bd = sdesc(sQ + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024);
+          umma_ss(tmem + C::S_COL, ad, bd, idS, k > 0 ? 1u : 0u);
+        }
+      };
+      if (ok) {
+        ok = mbar_wait(ring_full(0), 0, abort_flag, a.ws, 0x202);
+        if (ok) {
+          tc_fence_after();
+          issue_S(0);
+          umma_commit(s_full);
+          umma_commit(ring_empty(0));
+          if (ntiles == 1 || nxt.h != cur.h) umma_commit(q_empty);
+          e = 1;
+        }
+      }
+      for (int li = 0; li < ntiles && ok; ++li) {
+        if (li + 1 < ntiles) {
+          if (nxt.h != cur.h) {
+            ++hc;
+            ok = mbar_wait(q_full, hc & 1, abort_flag, a.ws, 0x203);
+            if (!ok) break;
+          }
+          ok = mbar_wait(s_empty, li & 1, abort_flag, a.ws, 0x204);
+          if (!ok) break;
+          const int s = int(e % C::NSLOT);
+          ok = mbar_wait(ring_full(s), (e / C::NSLOT) & 1, abort_flag, a.ws, 0x205);
+          if (!ok) break;
+          tc_fence_after();
+          issue_S(uint32_t(s));
+          umma_commit(s_full);
+          umma_commit(ring_empty(s));
+          ++e;
+          // last S of this head: Q may be replaced once it completes
+          const int h_now = nxt.h;
+          nxt.next();
+          if (li + 2 >= ntiles || nxt.h != h_now) umma_commit(q_empty);
+        }
+        // aggregation of tile li
+        ok = mbar_wait(w_full, li & 1, abort_flag, a.ws, 0x206);
+        if (!ok) break;
+        const int s = int(e % C::NSLOT);
+        ok = mbar_wait(ring_full(s), (e / C::NSLOT) & 1, abort_flag, a.ws, 0x207);
+        if (!ok) break;
+        if (cur.seg_first && sc > 0) {
+          ok = mbar_wait(o_empty, (sc - 1) & 1, abort_flag, a.ws, 0x208);
+          if (!ok) break;
+        }
+        tc_fence_after();
+        const uint32_t vaddr = sRing + s * C::KV_TILE;
+#pragma unroll
+        for (int k = 0; k < T / 16; ++k) {
+          const uint32_t acc = (cur.seg_first && k == 0) ? 0u : 1u;
+          if (C::TRANS) {
+            // O^T[d, p] += sum_t V[t, d] A[t, p]:  A-operand V^T (MN-major), B-operand A (MN-major)
+            const uint64_t ad = sdesc(vaddr + k * 2048, T * 128, 1024);
+            const uint64_t bd = sdesc(sW + k * 2048, T * 128, 1024);
+            umma_ss(tmem + C::O_COL, ad, bd, idO, acc);
+          } else {
+#pragma unroll
+            for (int mb = 0; mb < PS / 128; ++mb) {
+              // O[p, d] += sum_t A[t, p] V[t, d]: A-operand A^T (MN-major), B-operand V (MN-major)
+              const uint64_t ad = sdesc(sW + mb * 2 * (T * 128) + k * 2048, T * 128, 1024);
+              const uint64_t bd = sdesc(vaddr + k * 2048, T * 128, 1024);
+              umma_ss(tmem + C::O_COL + mb * D, ad, bd, idO, acc);
+            }
+          }
+        }
+        umma_commit(w_empty);
+        umma_commit(ring_empty(s));
+        ++e;
+        if (cur.seg_last) {
+          umma_commit(o_full);
+          ++sc;
+        }
+        cur.next();
+      }
+      // make sure no UMMA is still running when TMEM is released
+      umma_commit(drain);
+      mbar_wait_bounded(drain, 0, 200000000ull);
+    } else if (warp >= kSoftWarp0) {
+      // ------------------------------------------- softmax + epilogue warps
+      const int sw = (warp - kSoftWarp0) >> 2;  // warpgroup: prototype half
+      const int q = warp & 3;                   // TMEM lane quadrant
+      const int row = 32 * q + lane;            // token within the tile
+      const uint32_t lane_off = uint32_t(32 * q) << 16;
+      const float c2 = a.scale * 1.4426950408889634f;  // scale * log2(e)
+      float2* stats = reinterpret_cast<float2*>(smem + C::OFF_STATS);
+      TileWalker cur(a, tb, te, T);
+      int seg_idx = 0;
+      bool ok = true;
+      // every wait result is made warp-uniform so a timeout never splits a warp
+      auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
+      };
+      for (int li = 0; li < ntiles && ok; ++li) {
+        ok = wwait(s_full, li & 1, 0x301);
+        if (!ok) break;
+        tc_fence_after();
+        float v[C::HALF];
+#pragma unroll
+        for (int c = 0; c < C::HALF / 32; ++c) tmem_ld32(tmem + lane_off + C::S_COL + sw * C::HALF + 32 * c, v + 32 * c);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(s_empty);
+        const bool valid = row < cur.n;
+        const int64_t tok = cur.tok0 + row;
+        if (MODE == kFused) {
+          float m = v[0];
+#pragma unroll
+          for (int j = 1; j < C::HALF; ++j) m = fmaxf(m, v[j]);
+          const float mc = m * c2;
+          float z = 0.f;
+#pragma unroll
+          for (int j = 0; j < C::HALF; ++j) {
+            v[j] = ex2(fmaf(v[j], c2, -mc));
+            z += v[j];
+          }
+          // exchange (max, sum) with the other warpgroup's thread of this token
+          if (li > 0) {
+            ok = wwait(st_used, (li - 1) & 1, 0x304);
+            if (!ok) break;
+          }
+          stats[sw * T + row] = make_float2(m, z);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(st_ready);
+          ok = wwait(st_ready, li & 1, 0x305);
+          if (!ok) break;
+          const float2 o = stats[(1 - sw) * T + row];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(st_used);
+          const float M = fmaxf(m, o.x);
+          const float f_self = ex2((m - M) * c2), f_other = ex2((o.x - M) * c2);
+          const float Z = z * f_self + o.y * f_other;
+          const float f = f_self / Z;
+#pragma unroll
+          for (int j = 0; j < C::HALF; ++j) v[j] *= f;
+          if (sw == 0 && valid && lse_out) lse_out[tok * a.H + cur.h] = M * a.scale + logf(Z);
+        } else {
+          const float L2 = valid ? lse_in[tok * a.H + cur.h] * 1.4426950408889634f : 0.f;
+#pragma unroll
+          for (int j = 0; j < C::HALF; ++j) v[j] = ex2(fmaf(v[j], c2, -L2));
+        }
+        if (!valid) {
+#pragma unroll
+          for (int j = 0; j < C::HALF; ++j) v[j] = 0.f;
+        }
+        if (li > 0) {
+          ok = wwait(w_empty, (li - 1) & 1, 0x302);
+          if (!ok) break;
+        }
+        // weights -> shared memory, [PS/64 blocks][128 tokens][64 prototypes], 128-byte swizzle
+        uint8_t* wrow = smem + C::OFF_W + row * 128;
+#pragma unroll
+        for (int k = 0; k < C::HALF / 8; ++k) {
+          const int p = sw * C::HALF + 8 * k;
+          const int blk = p >> 6, chunk = (p & 63) >> 3;
+          uint4 pk;
+          pk.x = pack_bf16(v[8 * k + 0], v[8 * k + 1]);
+          pk.y = pack_bf16(v[8 * k + 2], v[8 * k + 3]);
+          pk.z = pack_bf16(v[8 * k + 4], v[8 * k + 5]);
+          pk.w = pack_bf16(v[8 * k + 6], v[8 * k + 7]);
+          *reinterpret_cast<uint4*>(wrow + blk * (T * 128) + ((chunk ^ (row & 7)) << 4)) = pk;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(w_full);
+        if (cur.seg_last) {
+          ok = wwait(o_full, seg_idx & 1, 0x303);
+          if (!ok) break;
+          tc_fence_after();
+          const bool whole = cur.seg0 >= tb && cur.seg1 <= te;
+          float* dst = whole ? sketch + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D
+                             : a.partial + ((int64_t(wk) * 2 + partial_slot(total, W, wk, cur.seg0)) * a.P + p0) * D;
+          store_sketch<D, PS, C::TRANS, C::O_COL>(tmem, lane_off, sw, q, lane, dst);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(o_empty);
+          ++seg_idx;
+        }
+        cur.next();
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ lse only
+// Per-token log-sum-exp over all P prototypes, P in chunks of NC <= 256
+// (two TMEM buffers of NC columns alternate over (tile, chunk)).
+template <int D, int NC, int NCH>
+struct LseCfg {
+  static constexpr int P = NC * NCH;
+  static constexpr int KV_TILE = T * D * 2;
+  static constexpr int Q_BYTES = P * D * 2;
+  static constexpr int NSLOT = (Q_BYTES + 4 * KV_TILE <= 200 * 1024) ? 4 : 3;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_RING = Q_BYTES;
+  static constexpr int OFF_STATS = OFF_RING + NSLOT * KV_TILE;
+  static constexpr int OFF_BAR = OFF_STATS + 2 * T * 8;
+  static constexpr int NBAR = 2 * NSLOT + 9;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+  static constexpr int SMEM = OFF_MISC + 16;
+  static constexpr int TMEM_COLS = tmem_cols_for(2 * NC);
+  static constexpr int HALF = NC / 2;
+};
+
+template <int D, int NC, int NCH>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_lse_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ, Args a,
+                  float* __restrict__ lse_out) {
+  using C = LseCfg<D, NC, NCH>;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (ws_failed(a.ws)) return;
+  if (smem_u32(smem) & 1023u) {
+    if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xA12u);
+    return;
+  }
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t sQ = sbase + C::OFF_Q, sRing = sbase + C::OFF_RING;
+  const uint32_t bar0 = sbase + C::OFF_BAR;
+  auto ring_full = [&](int s) { return bar0 + 8u * s; };
+  auto ring_empty = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
+  const uint32_t q_full = bar0 + 8u * (2 * C::NSLOT), q_empty = q_full + 8, s_full0 = q_full + 16,
+                 s_empty0 = q_full + 32, drain = q_full + 48, st_ready = q_full + 56, st_used = q_full + 64;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+  const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
+  const int64_t total = tph * a.H;
+  const int W = gridDim.x, wk = blockIdx.x;
+  const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
+  const int ntiles = int(te - tb);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(ring_full(s), 1);
+      mbar_init(ring_empty(s), 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    mbar_init(s_full0, 1);
+    mbar_init(s_full0 + 8, 1);
+    mbar_init(s_empty0, kSoftWarps);
+    mbar_init(s_empty0 + 8, kSoftWarps);
+    mbar_init(drain, 1);
+    mbar_init(st_ready, kSoftWarps);
+    mbar_init(st_used, kSoftWarps);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (ntiles > 0) {
+    if (warp == 0 && lane == 0) {
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmQ);
+      TileWalker it(a, tb, te, T);
+      int hc = 0, prev_h = -1;
+      uint32_t e = 0;
+      bool ok = true;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        if (it.h != prev_h) {
+          if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0x111);
+          if (!ok) break;
+          mbar_arrive_expect_tx(q_full, C::Q_BYTES);
+#pragma unroll
+          for (int c = 0; c < NCH; ++c)
+#pragma unroll
+            for (int dh = 0; dh < D / 64; ++dh)
+              tma_load_3d(sQ + dh * C::P * 128 + c * NC * 128, &tmQ, q_full, 64 * dh, c * NC, it.h);
+          prev_h = it.h;
+          ++hc;
+        }
+        const int s = int(e % C::NSLOT);
+        if (e >= uint32_t(C::NSLOT)) ok = mbar_wait(ring_empty(s), ((e / C::NSLOT) + 1) & 1, abort_flag, a.ws, 0x112);
+        if (!ok) break;
+        mbar_arrive_expect_tx(ring_full(s), C::KV_TILE);
+#pragma unroll
+        for (int dh = 0; dh < D / 64; ++dh)
+          tma_load_3d(sRing + s * C::KV_TILE + dh * T * 128, &tmK, ring_full(s), 64 * dh, it.h, int(it.tok0));
+        ++e;
+        it.next();
+      }
+      if (!ok) {
+        for (uint32_t k = (e > uint32_t(C::NSLOT) ? e - C::NSLOT : 0); k < e; ++k)
+          mbar_wait_bounded(ring_full(int(k % C::NSLOT)), (k / C::NSLOT) & 1, 200000000ull);
+      }
+    } else if (warp == 1 && lane == 0) {
+      constexpr uint32_t idS = idesc_bf16(128, NC, 0, 0);
+      TileWalker cur(a, tb, te, T);
+      int hc = 0, prev_h = -1;
+      bool ok = true;
+      uint32_t g = 0;  // (tile, chunk) counter
+      for (int li = 0; li < ntiles && ok; ++li) {
+        const int h_now = cur.h;
+        if (h_now != prev_h) {
+          prev_h = h_now;
+          ok = mbar_wait(q_full, hc & 1, abort_flag, a.ws, 0x211);
+          ++hc;
+          if (!ok) break;
+        }
+        const int s = int(uint32_t(li) % C::NSLOT);
+        ok = mbar_wait(ring_full(s), (uint32_t(li) / C::NSLOT) & 1, abort_flag, a.ws, 0x212);
+        if (!ok) break;
+        const uint32_t kaddr = sRing + s * C::KV_TILE;
+        for (int c = 0; c < NCH && ok; ++c, ++g) {
+          const int buf = int(g & 1);
+          if (g >= 2) ok = mbar_wait(s_empty0 + 8 * buf, ((g >> 1) + 1) & 1, abort_flag, a.ws, 0x213);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) {
+            const uint64_t ad = sdesc(kaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024);
+            const uint64_t bd = sdesc(sQ + (k >> 2) * (C::P * 128) + c * NC * 128 + (k & 3) * 32, 16, 1024);
+            umma_ss(tmem + buf * NC, ad, bd, idS, k > 0 ? 1u : 0u);
+          }
+          umma_commit(s_full0 + 8 * buf);
+        }
+        if (!ok) break;
+        umma_commit(ring_empty(s));
+        cur.next();
+        if (li + 1 >= ntiles || cur.h != h_now) umma_commit(q_empty);
+      }
+      umma_commit(drain);
+      mbar_wait_bounded(drain, 0, 200000000ull);
+    } else if (warp >= kSoftWarp0) {
+      const int sw = (warp - kSoftWarp0) >> 2, q = warp & 3, row = 32 * q + lane;
+      const uint32_t lane_off = uint32_t(32 * q) << 16;
+      const float c2 = a.scale * 1.4426950408889634f;
+      float2* stats = reinterpret_cast<float2*>(smem + C::OFF_STATS);
+      TileWalker cur(a, tb, te, T);
+      bool ok = true;
+      uint32_t g = 0;
+      auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
+      };
+      for (int li = 0; li < ntiles && ok; ++li) {
+        float m = -INFINITY, z = 0.f;
+        for (int c = 0; c < NCH && ok; ++c, ++g) {
+          const int buf = int(g & 1);
+          ok = wwait(s_full0 + 8 * buf, (g >> 1) & 1, 0x311);
+          if (!ok) break;
+          tc_fence_after();
+          float v[C::HALF];
+#pragma unroll
+          for (int k = 0; k < C::HALF / 32; ++k) tmem_ld32(tmem + lane_off + buf * NC + sw * C::HALF + 32 * k, v + 32 * k);
+          tmem_ld_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(s_empty0 + 8 * buf);
+          float mm = v[0];
+#pragma unroll
+          for (int j = 1; j < C::HALF; ++j) mm = fmaxf(mm, v[j]);
+          const float M = fmaxf(m, mm), Mc = M * c2;
+          float zz = 0.f;
+#pragma unroll
+          for (int j = 0; j < C::HALF; ++j) zz += ex2(fmaf(v[j], c2, -Mc));
+          z = z * ex2((m - M) * c2) + zz;
+          m = M;
+        }
+        if (!ok) break;
+        if (li > 0) {
+          ok = wwait(st_used, (li - 1) & 1, 0x312);
+          if (!ok) break;
+        }
+        stats[sw * T + row] = make_float2(m, z);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(st_ready);
+        ok = wwait(st_ready, li & 1, 0x313);
+        if (!ok) break;
+        const float2 o = stats[(1 - sw) * T + row];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(st_used);
+        if (sw == 0 && row < cur.n) {
+          const float M = fmaxf(m, o.x);
+          const float Z = z * ex2((m - M) * c2) + o.y * ex2((o.x - M) * c2);
+          lse_out[(cur.tok0 + row) * a.H + cur.h] = M * a.scale + logf(Z);
+        }
+        cur.next();
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------- host side
+template <int D, int PS, int MODE>
+static cudaError_t launch_fwd_t(const Args& a, int W, float* sketch, float* lse_out, const float* lse_in,
+                                cudaStream_t st) {
+  using C = Cfg<D, PS, MODE>;
+  CUtensorMap tk, tv, tq;
+  if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
+      !make_q_map(&tq, a.Q, a.H, a.P, D, PS))
+    return cudaErrorInvalidValue;
+  auto fn = &tc_fwd_kernel<D, PS, MODE>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  dim3 grid(W, a.P / PS);
+  fn<<<grid, kThreads, C::SMEM, st>>>(tk, tv, tq, a, sketch, lse_out, lse_in);
+  return cudaGetLastError();
+}
+
+template <int D, int NC, int NCH>
+static cudaError_t launch_lse_t(const Args& a, int W, float* lse_out, cudaStream_t st) {
+  using C = LseCfg<D, NC, NCH>;
+  CUtensorMap tk, tq;
+  if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_q_map(&tq, a.Q, a.H, a.P, D, NC)) return cudaErrorInvalidValue;
+  auto fn = &tc_lse_kernel<D, NC, NCH>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  fn<<<W, kThreads, C::SMEM, st>>>(tk, tq, a, lse_out);
+  return cudaGetLastError();
+}
+
+}  // namespace tcf
+
+// Shapes served by the tensor-core forward: bf16, d in {64, 128},
+// P in {128, 256} (one CTA holds all prototypes) or P = 512 (lse pass, then
+// two 256-prototype slices).
+bool tc_fwd_supported(int P, int d, sa_dtype dt) {
+  if (dt != SA_BF16 || (d != 64 && d != 128)) return false;
+  if (P != 128 && P != 256 && P != 512) return false;
+  return tcc::device_is_sm103() && tc_path_enabled();
+}
+
+// P = 512, or P = 256 with d = 128 (whose fused variant does not fit 227 KB of
+// shared memory next to the statistics exchange): lse pass, then slices of 256.
+bool tc_fwd_needs_lse_pass_d(int P, int d) { return P == 512 || (P == 256 && d == 128); }
+
+const char* tc_fwd_name(int P, int d) {
+  if (tc_fwd_needs_lse_pass_d(P, d)) return d == 128 ? "tc_fwd_kernel<128,256,sliced>" : "tc_fwd_kernel<64,256,sliced>";
+  if (P == 256) return "tc_fwd_kernel<64,256,fused>";
+  return d == 128 ? "tc_fwd_kernel<128,128,fused>" : "tc_fwd_kernel<64,128,fused>";
+}
+
+int tc_tile_tokens() { return tcc::T; }
+
+int tc_fwd_workers(int num_sms, int P, int) {
+  const int slices = P > 256 ? P / 256 : 1;
+  const int w = num_sms / slices;
+  return w < 1 ? 1 : w;
+}
+
+cudaError_t launch_tc_lse(const Args& a, float* lse, cudaStream_t st) {
+  if (a.N == 0) return cudaSuccess;
+  const int W = tcc::device_sm_count();
+  if (a.d == 128) {
+    if (a.P == 512) return tcf::launch_lse_t<128, 256, 2>(a, W, lse, st);
+    if (a.P == 256) return tcf::launch_lse_t<128, 256, 1>(a, W, lse, st);
+    if (a.P == 128) return tcf::launch_lse_t<128, 128, 1>(a, W, lse, st);
+  } else {
+    if (a.P == 512) return tcf::launch_lse_t<64, 256, 2>(a, W, lse, st);
+    if (a.P == 256) return tcf::launch_lse_t<64, 256, 1>(a, W, lse, st);
+    if (a.P == 128) return tcf::launch_lse_t<64, 128, 1>(a, W, lse, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_tc_fwd(const Args& a, int W, float* sketch, float* lse, cudaStream_t st) {
+  if (a.N == 0) return cudaSuccess;
+  using namespace tcf;
+  if (tc_fwd_needs_lse_pass_d(a.P, a.d))  // lse (from launch_tc_lse beforehand) is an input here
+    return a.d == 128 ? launch_fwd_t<128, 256, kSliced>(a, W, sketch, nullptr, lse, st)
+                      : launch_fwd_t<64, 256, kSliced>(a, W, sketch, nullptr, lse, st);
+  if (a.P == 256) return launch_fwd_t<64, 256, kFused>(a, W, sketch, lse, nullptr, st);
+  return a.d == 128 ? launch_fwd_t<128, 128, kFused>(a, W, sketch, lse, nullptr, st)
+                    : launch_fwd_t<64, 128, kFused>(a, W, sketch, lse, nullptr, st);
+}
 
 }  // namespace sa

@@ -1,0 +1,31 @@
+"""The tensor-core kernels against the CUDA-core kernels on the same inputs
+(two independent GPU implementations of Sec. 3.1), plus which kernel runs."""
+import pytest
+import torch
+
+import harness
+from paper_2609_08443_gb300 import binding, workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("P,d", [(128, 64), (256, 64), (128, 128), (256, 128), (512, 128), (512, 64)])
+def test_tensor_core_path_matches_cuda_core_path(cuda_lib, P, d):
+    spec = wl.custom([700, 0, 128, 129, 3000, 1], H=2, P=P, d=d, dtype=wl.BF16, seed=P * 7 + d)
+    host = wl.make_host(spec)
+    t = wl.host_to_torch(spec, host, torch.device("cuda"))
+    assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, False).startswith("tc_")
+    tc = harness.gpu_outputs(spec, t, bwd=True)
+    binding.sa_select_path(1)
+    try:
+        assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, False).startswith("simt")
+        simt = harness.gpu_outputs(spec, t, bwd=True)
+    finally:
+        binding.sa_select_path(0)
+    for k in ("sketch", "dK", "dV", "dQ"):
+        assert harness.rel_err(tc[k], simt[k]) <= 2e-2, k
+    assert abs(tc["lse"] - simt["lse"]).max() <= 5e-3 * max(1.0, abs(simt["lse"]).max())
+
+
+def test_fp32_uses_cuda_cores(cuda_lib):
+    assert binding.sa_main_kernel_name(64, 64, binding.SA_F32, False).startswith("simt")
