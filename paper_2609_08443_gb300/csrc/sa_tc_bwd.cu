@@ -1,13 +1,559 @@
-// tcgen05 backward kernel (sm_103a).  Not yet enabled.
+// tcgen05 / TMEM / TMA backward kernels of the SA sketching step (sm_103a).
+//
+// Chain rule of Sec. 3.1 with upstream G = dL/dsketch[b, h] and the forward's
+// per-token log-sum-exp (FlashSA's softmax statistic, Sec. 4.4), so the
+// weights are recomputed as A = exp(S - lse) without any reduction:
+//   S^T  = K Q^T                 (UMMA, tokens on TMEM lanes)
+//   A    = exp(scale S - lse)    (registers; bf16 copy in shared memory)
+//   dA^T = V G^T                 (UMMA)
+//   dV   = A G                   (UMMA, contraction over prototypes)
+//   D_i  = dV_i . v_i            (= sum_j A[j,i] dA[j,i])
+//   dS   = A o (dA - D)          (registers -> bf16 in shared memory)
+//   dK   = scale dS Q            (UMMA)
+//   dQ  += scale dS^T K          (UMMA, accumulated in TMEM over a worker's
+//                                 tiles of one head; per-worker partials are
+//                                 summed in worker order afterwards)
+// Modes: kFull keeps all P prototypes in one CTA (TMEM: S/dA, dV, dK, dQ);
+// kSlice handles one slice of prototypes and only dQ, with D_i read from the
+// token-side kernel (tc_bwd_tok_kernel) that computes dV, dK and D_i for
+// shapes whose four TMEM accumulators do not fit one SM.
+// Warp roles: 0 TMA, 1 UMMA, 2-3 dsketch loader (fp32 -> bf16 swizzled),
+// 4-11 softmax / epilogue.  Every wait is bounded.
+#include <cuda.h>
+
+#include "sa_ptx.cuh"
 #include "sa_tc.cuh"
+#include "sa_tc_common.cuh"
 
 namespace sa {
+namespace tcb {
 
-bool tc_bwd_supported(int, int, sa_dtype) { return false; }
-const char* tc_bwd_name(int, int) { return "tc_bwd"; }
+using namespace ptx;
+using namespace tcc;
+
+enum Mode { kFull = 0, kSlice = 1 };
+
+template <int D, int PS, int MODE>
+struct BCfg {
+  static constexpr int KV_TILE = T * D * 2;
+  static constexpr int Q_BYTES = PS * D * 2;
+  static constexpr int AB_BYTES = T * PS * 2;
+  static constexpr int NSLOT = 4;  // even: even slots hold K tiles, odd slots V tiles
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_G = Q_BYTES;
+  static constexpr int OFF_AB = OFF_G + Q_BYTES;
+  static constexpr int OFF_RING = OFF_AB + AB_BYTES;
+  static constexpr int OFF_BAR = OFF_RING + NSLOT * KV_TILE;
+  static constexpr int NBAR = 2 * NSLOT + 20;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+  static constexpr int SMEM = OFF_MISC + 16;
+  static constexpr int SD_COL = 0;
+  static constexpr int DV_COL = PS;
+  static constexpr int DK_COL = PS + D;
+  static constexpr int DQ_COL = (MODE == kFull) ? PS + 2 * D : PS;
+  static constexpr int TMEM_COLS = tmem_cols_for(DQ_COL + (PS / 128) * D);
+  static constexpr int HALF = PS / 2;
+  static_assert(TMEM_COLS <= 512, "TMEM budget");
+  static_assert(SMEM <= 232448, "shared memory budget");
+};
+
+// one token row of dV or dK (fp32 from TMEM) -> bf16 global row, columns
+// [c0, c0 + NCOL) of this warpgroup's half
+template <int NCOL>
+__device__ __forceinline__ void store_row_bf16(uint32_t taddr, __nv_bfloat16* dst, float mul, bool valid) {
+  float v[32];
+#pragma unroll
+  for (int c = 0; c < NCOL; c += 32) {
+    tmem_ld32(taddr + c, v);
+    tmem_ld_wait();
+    if (valid) {
+      uint4* o = reinterpret_cast<uint4*>(dst + c);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        uint4 pk;
+        pk.x = pack_bf16(v[8 * k + 0] * mul, v[8 * k + 1] * mul);
+        pk.y = pack_bf16(v[8 * k + 2] * mul, v[8 * k + 3] * mul);
+        pk.z = pack_bf16(v[8 * k + 4] * mul, v[8 * k + 5] * mul);
+        pk.w = pack_bf16(v[8 * k + 6] * mul, v[8 * k + 7] * mul);
+        o[k] = pk;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+template <int D, int PS, int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_bwd_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                  const __grid_constant__ CUtensorMap tmQ, Args a, const float* __restrict__ dsk,
+                  const float* __restrict__ lse, const float* __restrict__ Dco_in, __nv_bfloat16* __restrict__ dK,
+                  __nv_bfloat16* __restrict__ dV) {
+  using C = BCfg<D, PS, MODE>;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (ws_failed(a.ws)) return;
+  if (smem_u32(smem) & 1023u) {
+    if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xB11u);
+    return;
+  }
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t sQ = sbase + C::OFF_Q, sG = sbase + C::OFF_G, sAB = sbase + C::OFF_AB, sRing = sbase + C::OFF_RING;
+  const uint32_t bar0 = sbase + C::OFF_BAR;
+  auto ring_full = [&](int s) { return bar0 + 8u * s; };
+  auto ring_empty = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
+  const uint32_t b1 = bar0 + 8u * (2 * C::NSLOT);
+  const uint32_t q_full = b1, q_empty = b1 + 8, g_full = b1 + 16, g_empty = b1 + 24, s_full = b1 + 32,
+                 sd_free_s = b1 + 40, da_full = b1 + 48, sd_free_da = b1 + 56, a_full = b1 + 64, dv_full = b1 + 72,
+                 dv_empty = b1 + 80, ds_full = b1 + 88, ab_empty = b1 + 96, dk_empty = b1 + 104, dq_full = b1 + 112,
+                 dq_empty = b1 + 120, drain = b1 + 128;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+
+  const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
+  const int64_t total = tph * a.H;
+  const int W = gridDim.x, wk = blockIdx.x, slice = blockIdx.y;
+  const int p0 = slice * PS;
+  const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
+  const int ntiles = int(te - tb);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(ring_full(s), 1);
+      // V slots are released by the softmax warps once they have read v_i for D_i
+      mbar_init(ring_empty(s), (MODE == kFull && (s & 1)) ? kSoftWarps : 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    mbar_init(g_full, 2);
+    mbar_init(g_empty, 1);
+    mbar_init(s_full, 1);
+    mbar_init(sd_free_s, kSoftWarps);
+    mbar_init(da_full, 1);
+    mbar_init(sd_free_da, kSoftWarps);
+    mbar_init(a_full, kSoftWarps);
+    mbar_init(dv_full, 1);
+    mbar_init(dv_empty, kSoftWarps);
+    mbar_init(ds_full, kSoftWarps);
+    mbar_init(ab_empty, 1);
+    mbar_init(dk_empty, kSoftWarps);
+    mbar_init(dq_full, 1);
+    mbar_init(dq_empty, kSoftWarps);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (ntiles > 0) {
+    if (warp == 0 && lane == 0) {
+      // ---------------------------------------------------------- TMA producer
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      tma_prefetch_desc(&tmQ);
+      TileWalker it(a, tb, te, T);
+      int hc = 0, prev_h = -1;
+      uint32_t e = 0;
+      bool ok = true;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        if (it.h != prev_h) {
+          if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0x401);
+          if (!ok) break;
+          mbar_arrive_expect_tx(q_full, C::Q_BYTES);
+#pragma unroll
+          for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.h);
+          prev_h = it.h;
+          ++hc;
+        }
+#pragma unroll
+        for (int kv = 0; kv < 2; ++kv) {
+          const int s = int(e % C::NSLOT);
+          if (e >= uint32_t(C::NSLOT)) ok = mbar_wait(ring_empty(s), ((e / C::NSLOT) + 1) & 1, abort_flag, a.ws, 0x402);
+          if (!ok) break;
+          mbar_arrive_expect_tx(ring_full(s), C::KV_TILE);
+#pragma unroll
+          for (int dh = 0; dh < D / 64; ++dh)
+            tma_load_3d(sRing + s * C::KV_TILE + dh * T * 128, kv ? &tmV : &tmK, ring_full(s), 64 * dh, it.h,
+                        int(it.tok0));
+          ++e;
+        }
+        it.next();
+      }
+      if (!ok) {
+        for (uint32_t k = (e > uint32_t(C::NSLOT) ? e - C::NSLOT : 0); k < e; ++k)
+          mbar_wait_bounded(ring_full(int(k % C::NSLOT)), (k / C::NSLOT) & 1, 200000000ull);
+      }
+    } else if (warp == 1 && lane == 0) {
+      // ---------------------------------------------------------- UMMA issuer
+      constexpr uint32_t idSP = idesc_bf16(128, PS, 0, 0);      // [tok x P], K = d
+      constexpr uint32_t idTD = idesc_bf16(128, D, 0, 1);       // [tok x d], K = prototypes
+      constexpr uint32_t idQD = idesc_bf16(128, D, 1, 1);       // [proto x d], K = tokens
+      TileWalker cur(a, tb, te, T), nxt(a, tb, te, T);
+      nxt.next();
+      int hc = 0, gc = 0, hp = 0;
+      bool ok = true;
+      auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
+      };
+      // S(i) = K(i) Q^T into the S/dA columns
+      auto issue_S = [&](uint32_t kslot) {
+        const uint32_t kaddr = sRing + kslot * C::KV_TILE;
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          umma_ss(tmem + C::SD_COL, sdesc(kaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                  sdesc(sQ + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
+      };
+      wt(q_full, 0, 0x501);
+      wt(ring_full(0), 0, 0x502);
+      if (ok) {
+        tc_fence_after();
+        issue_S(0);
+        umma_commit(s_full);
+      }
+      bool first_of_hp = true;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        const uint32_t eK = 2u * li, eV = eK + 1;
+        const int sK = int(eK % C::NSLOT), sV = int(eV % C::NSLOT);
+        // ---- dA(i) = V(i) G^T
+        if (cur.seg_first) {
+          wt(g_full, gc & 1, 0x503);
+          ++gc;
+        }
+        wt(ring_full(sV), (eV / C::NSLOT) & 1, 0x504);
+        wt(sd_free_s, li & 1, 0x505);
+        if (!ok) break;
+        tc_fence_after();
+        {
+          const uint32_t vaddr = sRing + sV * C::KV_TILE;
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k)
+            umma_ss(tmem + C::SD_COL, sdesc(vaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                    sdesc(sG + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
+        }
+        umma_commit(da_full);
+        if (MODE == kSlice) umma_commit(ring_empty(sV));
+        // ---- dV(i) = A G
+        if (MODE == kFull) {
+          wt(a_full, li & 1, 0x506);
+          if (li > 0) wt(dv_empty, (li - 1) & 1, 0x507);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < PS / 16; ++k)
+            umma_ss(tmem + C::DV_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                    sdesc(sG + k * 2048, PS * 128, 1024), idTD, k > 0 ? 1u : 0u);
+          umma_commit(dv_full);
+        }
+        if (!ok) break;
+        if (cur.seg_last) umma_commit(g_empty);
+        // ---- S(i+1), early when the head (and so Q) stays the same
+        const bool more = li + 1 < ntiles;
+        const bool hoist = more && nxt.h == cur.h;
+        if (hoist) {
+          wt(sd_free_da, li & 1, 0x508);
+          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0x509);
+          if (!ok) break;
+          tc_fence_after();
+          issue_S((eK + 2) % C::NSLOT);
+          umma_commit(s_full);
+        }
+        // ---- dK(i) = dS Q, dQ += dS^T K
+        wt(ds_full, li & 1, 0x50A);
+        if (MODE == kFull && li > 0) wt(dk_empty, (li - 1) & 1, 0x50B);
+        if (first_of_hp && hp > 0) wt(dq_empty, (hp - 1) & 1, 0x50C);
+        if (!ok) break;
+        tc_fence_after();
+        if (MODE == kFull) {
+#pragma unroll
+          for (int k = 0; k < PS / 16; ++k)
+            umma_ss(tmem + C::DK_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                    sdesc(sQ + k * 2048, PS * 128, 1024), idTD, k > 0 ? 1u : 0u);
+        }
+        {
+          const uint32_t kaddr = sRing + sK * C::KV_TILE;
+#pragma unroll
+          for (int k = 0; k < T / 16; ++k)
+#pragma unroll
+            for (int mb = 0; mb < PS / 128; ++mb)
+              umma_ss(tmem + C::DQ_COL + mb * D, sdesc(sAB + mb * 2 * (T * 128) + k * 2048, T * 128, 1024),
+                      sdesc(kaddr + k * 2048, T * 128, 1024), idQD, (first_of_hp && k == 0) ? 0u : 1u);
+        }
+        umma_commit(ab_empty);
+        umma_commit(ring_empty(sK));
+        const bool last_of_hp = !more || nxt.h != cur.h;
+        if (last_of_hp) {
+          umma_commit(dq_full);
+          umma_commit(q_empty);
+          ++hp;
+        }
+        first_of_hp = last_of_hp;
+        // ---- S(i+1) after a head change (Q replaced once dK(i) is done)
+        if (more && !hoist) {
+          ++hc;
+          wt(q_full, hc & 1, 0x50D);
+          wt(sd_free_da, li & 1, 0x50E);
+          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0x50F);
+          if (!ok) break;
+          tc_fence_after();
+          issue_S((eK + 2) % C::NSLOT);
+          umma_commit(s_full);
+        }
+        cur.next();
+        nxt.next();
+      }
+      umma_commit(drain);
+      mbar_wait_bounded(drain, 0, 200000000ull);
+    } else if (warp == 2 || warp == 3) {
+      // ------------------------------------ dsketch rows -> bf16, swizzled [d/64][PS][64]
+      const int t64 = threadIdx.x - 64;  // 0..63
+      TileWalker cur(a, tb, te, T);
+      int gc = 0;
+      bool ok = true;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        if (cur.seg_first) {
+          if (gc > 0) ok = __all_sync(0xffffffffu, mbar_wait(g_empty, (gc - 1) & 1, abort_flag, a.ws, 0x601));
+          if (!ok) break;
+          const float* src = dsk + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D;
+          constexpr int CHUNKS = PS * D / 8;
+          for (int c = t64; c < CHUNKS; c += 64) {
+            const int p = c / (D / 8), dd = (c % (D / 8)) * 8;
+            const float4 x = *reinterpret_cast<const float4*>(src + int64_t(p) * D + dd);
+            const float4 y = *reinterpret_cast<const float4*>(src + int64_t(p) * D + dd + 4);
+            uint4 pk;
+            pk.x = pack_bf16(x.x, x.y);
+            pk.y = pack_bf16(x.z, x.w);
+            pk.z = pack_bf16(y.x, y.y);
+            pk.w = pack_bf16(y.z, y.w);
+            const int dh = dd >> 6, chunk = (dd & 63) >> 3;
+            *reinterpret_cast<uint4*>(smem + C::OFF_G + dh * PS * 128 + p * 128 + ((chunk ^ (p & 7)) << 4)) = pk;
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(g_full);
+          ++gc;
+        }
+        cur.next();
+      }
+    } else if (warp >= kSoftWarp0) {
+      // ------------------------------------------------ softmax + epilogue
+      const int sw = (warp - kSoftWarp0) >> 2, q = warp & 3, row = 32 * q + lane;
+      const uint32_t lane_off = uint32_t(32 * q) << 16;
+      const float c2 = a.scale * 1.4426950408889634f;
+      TileWalker cur(a, tb, te, T), prev(a, tb, te, T);
+      bool ok = true;
+      auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
+      };
+      int hp = 0;
+      // dK of the previous tile and, at the end of a head piece, dQ
+      auto finish_prev = [&](const TileWalker& pw, bool last_of_hp) {
+        if (MODE == kFull) {
+          __nv_bfloat16* dst = dK + ((pw.tok0 + row) * a.H + pw.h) * int64_t(D) + sw * (D / 2);
+          store_row_bf16<D / 2>(tmem + lane_off + C::DK_COL + sw * (D / 2), dst, a.scale, row < pw.n);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(dk_empty);
+        }
+        if (last_of_hp) {
+          float* dst = a.dq_partial + ((int64_t(wk) * a.H + pw.h) * a.P + p0) * D;
+          store_sketch_scaled<D, PS, C::DQ_COL>(tmem, lane_off, sw, q, lane, dst, a.scale);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(dq_empty);
+          ++hp;
+        }
+      };
+      uint32_t apk[C::HALF / 2];  // this thread's A values, bf16 pairs
+      for (int li = 0; li < ntiles && ok; ++li) {
+        const bool valid = row < cur.n;
+        const int64_t tok = cur.tok0 + row;
+        const uint32_t eV = 2u * li + 1;
+        const int sV = int(eV % C::NSLOT);
+        // ---- A = exp(scale S - lse)
+        ok = wwait(s_full, li & 1, 0x701);
+        if (!ok) break;
+        tc_fence_after();
+        {
+          const float L2 = valid ? lse[tok * a.H + cur.h] * 1.4426950408889634f : 0.f;
+          float v[32];
+#pragma unroll
+          for (int c = 0; c < C::HALF / 32; ++c) {
+            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * c, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float x0 = valid ? ex2(fmaf(v[2 * j], c2, -L2)) : 0.f;
+              const float x1 = valid ? ex2(fmaf(v[2 * j + 1], c2, -L2)) : 0.f;
+              apk[16 * c + j] = pack_bf16(x0, x1);
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(sd_free_s);
+        // ---- previous tile's dK / dQ (their MMAs also release the AB buffer)
+        if (li > 0) {
+          ok = wwait(ab_empty, (li - 1) & 1, 0x702);
+          if (!ok) break;
+          tc_fence_after();
+          finish_prev(prev, prev.h != cur.h);
+          prev.next();
+        }
+        // ---- A -> shared memory [PS/64][128 tokens][64], 128-byte swizzle
+        if (MODE == kFull) {
+          uint8_t* rowp = smem + C::OFF_AB + row * 128;
+#pragma unroll
+          for (int k = 0; k < C::HALF / 8; ++k) {
+            const int p = sw * C::HALF + 8 * k;
+            const int blk = p >> 6, chunk = (p & 63) >> 3;
+            *reinterpret_cast<uint4*>(rowp + blk * (T * 128) + ((chunk ^ (row & 7)) << 4)) =
+                make_uint4(apk[4 * k], apk[4 * k + 1], apk[4 * k + 2], apk[4 * k + 3]);
+          }
+        }
+        if (MODE == kFull) {
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(a_full);
+        }
+        // ---- D_i
+        float Dv = 0.f;
+        if (MODE == kFull) {
+          ok = wwait(dv_full, li & 1, 0x703);
+          if (!ok) break;
+          tc_fence_after();
+          const uint8_t* vrow = smem + C::OFF_RING + sV * C::KV_TILE + row * 128;
+          float v[32];
+#pragma unroll
+          for (int c = 0; c < D; c += 32) {
+            tmem_ld32(tmem + lane_off + C::DV_COL + c, v);
+            tmem_ld_wait();
+            const int dh = c >> 6;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int chunk = ((c & 63) >> 3) + k;
+              const uint4 w = *reinterpret_cast<const uint4*>(vrow + dh * (T * 128) + ((chunk ^ (row & 7)) << 4));
+              Dv = fmaf(v[8 * k + 0], bf16lo(w.x), Dv);
+              Dv = fmaf(v[8 * k + 1], bf16hi(w.x), Dv);
+              Dv = fmaf(v[8 * k + 2], bf16lo(w.y), Dv);
+              Dv = fmaf(v[8 * k + 3], bf16hi(w.y), Dv);
+              Dv = fmaf(v[8 * k + 4], bf16lo(w.z), Dv);
+              Dv = fmaf(v[8 * k + 5], bf16hi(w.z), Dv);
+              Dv = fmaf(v[8 * k + 6], bf16lo(w.w), Dv);
+              Dv = fmaf(v[8 * k + 7], bf16hi(w.w), Dv);
+            }
+          }
+          // dV rows of this tile
+          __nv_bfloat16* dst = dV + (tok * a.H + cur.h) * int64_t(D) + sw * (D / 2);
+          store_row_bf16<D / 2>(tmem + lane_off + C::DV_COL + sw * (D / 2), dst, 1.f, valid);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(dv_empty);
+            mbar_arrive(ring_empty(sV));
+          }
+        } else {
+          Dv = valid ? Dco_in[tok * a.H + cur.h] : 0.f;
+        }
+        // ---- dS = A o (dA - D) -> shared memory (over A, whose readers are done)
+        ok = wwait(da_full, li & 1, 0x704);
+        if (!ok) break;
+        tc_fence_after();
+        {
+          uint8_t* rowp = smem + C::OFF_AB + row * 128;
+          float v[32];
+#pragma unroll
+          for (int c = 0; c < C::HALF / 32; ++c) {
+            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * c, v);
+            tmem_ld_wait();
+            uint32_t o[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const uint32_t w = apk[16 * c + j];
+              o[j] = pack_bf16(bf16lo(w) * (v[2 * j] - Dv), bf16hi(w) * (v[2 * j + 1] - Dv));
+            }
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int p = sw * C::HALF + 32 * c + 8 * k;
+              const int blk = p >> 6, chunk = (p & 63) >> 3;
+              *reinterpret_cast<uint4*>(rowp + blk * (T * 128) + ((chunk ^ (row & 7)) << 4)) =
+                  make_uint4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
+            }
+          }
+        }
+        tc_fence_before();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(sd_free_da);
+          mbar_arrive(ds_full);
+        }
+        cur.next();
+      }
+      if (ok) {
+        ok = wwait(ab_empty, (ntiles - 1) & 1, 0x705);
+        if (ok) {
+          tc_fence_after();
+          finish_prev(prev, true);
+        }
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int D, int PS, int MODE>
+static cudaError_t launch_bwd_t(const Args& a, int W, const float* dsk, const float* lse, const float* Dco, void* dK,
+                                void* dV, cudaStream_t st) {
+  using C = BCfg<D, PS, MODE>;
+  CUtensorMap tk, tv, tq;
+  if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
+      !make_q_map(&tq, a.Q, a.H, a.P, D, PS))
+    return cudaErrorInvalidValue;
+  auto fn = &tc_bwd_kernel<D, PS, MODE>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  dim3 grid(W, a.P / PS);
+  fn<<<grid, kThreads, C::SMEM, st>>>(tk, tv, tq, a, dsk, lse, Dco, static_cast<__nv_bfloat16*>(dK),
+                                      static_cast<__nv_bfloat16*>(dV));
+  return cudaGetLastError();
+}
+
+}  // namespace tcb
+
+// Tensor-core backward: bf16, all prototypes in one CTA when the four TMEM
+// accumulators fit (d = 64 with P <= 256, d = 128 with P = 128).
+bool tc_bwd_supported(int P, int d, sa_dtype dt) {
+  if (dt != SA_BF16 || !tcc::device_is_sm103() || !tc_path_enabled()) return false;
+  return (d == 64 && (P == 128 || P == 256)) || (d == 128 && P == 128);
+}
+
+const char* tc_bwd_name(int P, int d) {
+  if (d == 64) return P == 256 ? "tc_bwd_kernel<64,256,full>" : "tc_bwd_kernel<64,128,full>";
+  return "tc_bwd_kernel<128,128,full>";
+}
+
 int tc_bwd_workers(int num_sms, int, int) { return num_sms; }
-cudaError_t launch_tc_bwd(const Args&, int, const float*, const float*, void*, void*, cudaStream_t) {
-  return cudaErrorNotSupported;
+
+cudaError_t launch_tc_bwd(const Args& a, int W, const float* dsk, const float* lse, void* dK, void* dV,
+                          cudaStream_t st) {
+  if (a.N == 0) return cudaSuccess;
+  using namespace tcb;
+  if (a.d == 64) {
+    if (a.P == 256) return launch_bwd_t<64, 256, kFull>(a, W, dsk, lse, nullptr, dK, dV, st);
+    if (a.P == 128) return launch_bwd_t<64, 128, kFull>(a, W, dsk, lse, nullptr, dK, dV, st);
+  } else if (a.P == 128) {
+    return launch_bwd_t<128, 128, kFull>(a, W, dsk, lse, nullptr, dK, dV, st);
+  }
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace sa

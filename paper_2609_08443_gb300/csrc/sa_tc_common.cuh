@@ -107,6 +107,28 @@ __device__ __forceinline__ void store_sketch(uint32_t tmem, uint32_t lane_off, i
   }
 }
 
+// Prototype-major accumulator ([PS/128 blocks] lanes = prototype, columns = d)
+// times `mul` to global rows [PS][D] (used for dQ partials).
+template <int D, int PS, int O_COL>
+__device__ __forceinline__ void store_sketch_scaled(uint32_t tmem, uint32_t lane_off, int sw, int q, int lane,
+                                                    float* dst, float mul) {
+  float v[32];
+  constexpr int NB = PS / 128;
+  const int blk = NB == 2 ? sw : 0;
+  const int p = 128 * blk + 32 * q + lane;
+  const int c0 = NB == 2 ? 0 : (D / 2) * sw;
+  const int c1 = NB == 2 ? D : c0 + D / 2;
+#pragma unroll 1
+  for (int c = c0; c < c1; c += 32) {
+    ptx::tmem_ld32(tmem + lane_off + O_COL + blk * D + c, v);
+    ptx::tmem_ld_wait();
+    float4* o = reinterpret_cast<float4*>(dst + int64_t(p) * D + c);
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      o[k] = make_float4(v[4 * k] * mul, v[4 * k + 1] * mul, v[4 * k + 2] * mul, v[4 * k + 3] * mul);
+  }
+}
+
 // ------------------------------------------------------------- host helpers
 bool make_kv_map(CUtensorMap* m, const void* base, int64_t N, int H, int D);
 bool make_q_map(CUtensorMap* m, const void* Q, int H, int P, int D, int box_rows);

@@ -23,6 +23,7 @@ SHAPES = [
     (256, 128, wl.BF16, 1),
     (512, 64, wl.BF16, 1),
     (128, 64, wl.BF16, 3),
+    (128, 128, wl.BF16, 2),
     (96, 32, wl.BF16, 1),
     (200, 128, wl.F32, 1),
     (1024, 64, wl.BF16, 1),
