@@ -278,6 +278,18 @@ sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens,
     }
     l = scratch;
   }
+  if (plan.bwd_path == Path::TcBwd && sa::tc_bwd_split(P, d)) {
+    // token side (dV, dK, D_i) over all prototypes, then dQ per prototype slice
+    __nv_bfloat16* gbf = reinterpret_cast<__nv_bfloat16*>(base + plan.lay.gbf);
+    float* Dco = reinterpret_cast<float*>(base + plan.lay.dcoef);
+    const int Wq = sa::tc_bwd_dq_workers(sa::tcc::device_sm_count(), P);
+    SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tc_g_bf16(a, dsketch, gbf, st); }));
+    SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
+                  [&] { return sa::launch_tc_bwd_tok(a, plan.W_bwd, dsketch, gbf, l, Dco, dK, dV, st); }));
+    SA_TRY(launch(SA_KERNEL_BWD_MAIN, st, [&] { return sa::launch_tc_bwd_dq(a, Wq, dsketch, l, Dco, st); }));
+    SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, Wq, dQ, st); }));
+    return SA_OK;
+  }
   if (plan.bwd_path == Path::TcBwd) {
     SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
                   [&] { return sa::launch_tc_bwd(a, plan.W_bwd, dsketch, l, dK, dV, st); }));

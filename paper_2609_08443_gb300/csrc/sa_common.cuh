@@ -43,7 +43,8 @@ struct WsLayout {
   size_t partial;      // fp32 [W][2][P][d]: sketch pieces of cut segments
   size_t dq_partial;   // fp32 [W][H][P][d]: per-worker dQ per head (bwd)
   size_t lse;          // fp32 [N][H]: lse scratch when the caller passes none
-  size_t dcoef;        // fp32 [N][H]: D_i = dV_i . v_i (bwd, CUDA-core path)
+  size_t dcoef;        // fp32 [N][H]: D_i = dV_i . v_i (bwd)
+  size_t gbf;          // bf16 [B][H][P][d]: dsketch copy streamed by TMA (bwd, d = 128)
   size_t total;
 };
 
@@ -60,6 +61,8 @@ SA_HD WsLayout ws_layout(int B, int64_t N, int H, int P, int d, int W, bool bwd)
   off = align256(off + sizeof(float) * size_t(N) * size_t(H));
   L.dcoef = off;
   if (bwd) off = align256(off + sizeof(float) * size_t(N) * size_t(H));
+  L.gbf = off;
+  if (bwd && d == 128 && P > 128) off = align256(off + 2 * size_t(B) * size_t(H) * size_t(P) * size_t(d));
   L.total = off;
   return L;
 }

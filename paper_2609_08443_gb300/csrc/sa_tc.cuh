@@ -17,5 +17,13 @@ cudaError_t launch_tc_fwd(const Args& a, int W, float* sketch, float* lse, cudaS
 cudaError_t launch_tc_lse(const Args& a, float* lse, cudaStream_t st);
 cudaError_t launch_tc_bwd(const Args& a, int W, const float* dsk, const float* lse, void* dK, void* dV,
                           cudaStream_t st);
+// d = 128 with P in {256, 512}: token side (dV, dK, D_i) then prototype slices (dQ)
+bool tc_bwd_split(int P, int d);
+cudaError_t launch_tc_bwd_tok(const Args& a, int W, const float* dsk, __nv_bfloat16* gbf, const float* lse,
+                              float* Dco, void* dK, void* dV, cudaStream_t st);
+cudaError_t launch_tc_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
+                             cudaStream_t st);
+int tc_bwd_dq_workers(int num_sms, int P);
+cudaError_t launch_tc_g_bf16(const Args& a, const float* dsk, __nv_bfloat16* gbf, cudaStream_t st);
 
 }  // namespace sa

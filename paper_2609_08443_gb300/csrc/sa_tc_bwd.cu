@@ -533,11 +533,13 @@ static cudaError_t launch_bwd_t(const Args& a, int W, const float* dsk, const fl
 // accumulators fit (d = 64 with P <= 256, d = 128 with P = 128).
 bool tc_bwd_supported(int P, int d, sa_dtype dt) {
   if (dt != SA_BF16 || !tcc::device_is_sm103() || !tc_path_enabled()) return false;
-  return (d == 64 && (P == 128 || P == 256)) || (d == 128 && P == 128);
+  return (d == 64 && (P == 128 || P == 256)) || (d == 128 && (P == 128 || P == 256 || P == 512));
 }
 
 const char* tc_bwd_name(int P, int d) {
   if (d == 64) return P == 256 ? "tc_bwd_kernel<64,256,full>" : "tc_bwd_kernel<64,128,full>";
+  if (P == 512) return "tc_bwd_tok_kernel<128,512>";
+  if (P == 256) return "tc_bwd_tok_kernel<128,256>";
   return "tc_bwd_kernel<128,128,full>";
 }
 
@@ -554,6 +556,424 @@ cudaError_t launch_tc_bwd(const Args& a, int W, const float* dsk, const float* l
     return launch_bwd_t<128, 128, kFull>(a, W, dsk, lse, nullptr, dK, dV, st);
   }
   return cudaErrorInvalidValue;
+}
+
+}  // namespace sa
+
+// ===================================================================== tokens
+// Token side of the backward for shapes whose prototypes do not fit one CTA
+// (d = 128 with P > 128): all P prototypes pass through the CTA in chunks of
+// NC = 128 (Q and a bf16 copy of dsketch streamed by TMA), in one pass:
+//   dV_i   = sum_j A[j,i] G_j                   (UMMA, accumulates over chunks)
+//   u_i    = sum_j A[j,i] dA[j,i] Q_j            (UMMA on E = A o dA)
+//   qbar_i = sum_j A[j,i] Q_j                    (UMMA)
+//   D_i    = sum_j A[j,i] dA[j,i]                (registers)
+//   dK_i   = scale (u_i - D_i qbar_i)            (= scale sum_j dS[j,i] Q_j)
+// and D_i is written out for the prototype-side dQ kernel (kSlice mode above).
+namespace sa {
+namespace tcb {
+
+template <int D, int P>
+struct TokCfg {
+  static constexpr int NC = 128;
+  static constexpr int NCH = P / NC;
+  static constexpr int KV_TILE = T * D * 2;
+  static constexpr int QG_CHUNK = NC * D * 2;
+  static constexpr int NQG = 3;  // ring of Q / G chunks (entries alternate Q, G)
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = KV_TILE;
+  static constexpr int OFF_QG = 2 * KV_TILE;
+  static constexpr int OFF_AB = OFF_QG + NQG * QG_CHUNK;
+  static constexpr int OFF_EB = OFF_AB + T * NC * 2;
+  static constexpr int OFF_STATS = OFF_EB + T * NC * 2;
+  static constexpr int OFF_BAR = OFF_STATS + 2 * T * 4;
+  static constexpr int NBAR = 2 * NQG + 20;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+  static constexpr int SMEM = OFF_MISC + 16;
+  static constexpr int SD_COL = 0, DV_COL = NC, U_COL = NC + D, QB_COL = NC + 2 * D;
+  static constexpr int TMEM_COLS = tmem_cols_for(NC + 3 * D);
+  static constexpr int HALF = NC / 2;
+  static_assert(TMEM_COLS <= 512 && SMEM <= 232448, "budget");
+};
+
+template <int D, int P>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_bwd_tok_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                      const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmG, Args a,
+                      const float* __restrict__ lse, float* __restrict__ Dco, __nv_bfloat16* __restrict__ dK,
+                      __nv_bfloat16* __restrict__ dV) {
+  using C = TokCfg<D, P>;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (ws_failed(a.ws)) return;
+  if (smem_u32(smem) & 1023u) {
+    if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xB21u);
+    return;
+  }
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t sK = sbase + C::OFF_K, sV = sbase + C::OFF_V, sQG = sbase + C::OFF_QG, sAB = sbase + C::OFF_AB,
+                 sEB = sbase + C::OFF_EB;
+  const uint32_t bar0 = sbase + C::OFF_BAR;
+  auto qg_full = [&](int s) { return bar0 + 8u * s; };
+  auto qg_empty = [&](int s) { return bar0 + 8u * (C::NQG + s); };
+  const uint32_t b1 = bar0 + 8u * (2 * C::NQG);
+  const uint32_t k_full = b1, k_empty = b1 + 8, v_full = b1 + 16, v_empty = b1 + 24, s_full = b1 + 32,
+                 sd_free_s = b1 + 40, da_full = b1 + 48, sd_free_da = b1 + 56, a_full = b1 + 64, ab_empty = b1 + 72,
+                 e_full = b1 + 80, eb_empty = b1 + 88, acc_full = b1 + 96, acc_empty = b1 + 104, st_ready = b1 + 112,
+                 st_used = b1 + 120, drain = b1 + 128;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+  const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
+  const int64_t total = tph * a.H;
+  const int W = gridDim.x, wk = blockIdx.x;
+  const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
+  const int ntiles = int(te - tb);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NQG; ++s) {
+      mbar_init(qg_full(s), 1);
+      mbar_init(qg_empty(s), 1);
+    }
+    mbar_init(k_full, 1);
+    mbar_init(k_empty, 1);
+    mbar_init(v_full, 1);
+    mbar_init(v_empty, 1);
+    mbar_init(s_full, 1);
+    mbar_init(sd_free_s, kSoftWarps);
+    mbar_init(da_full, 1);
+    mbar_init(sd_free_da, kSoftWarps);
+    mbar_init(a_full, kSoftWarps);
+    mbar_init(ab_empty, 1);
+    mbar_init(e_full, kSoftWarps);
+    mbar_init(eb_empty, 1);
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, kSoftWarps);
+    mbar_init(st_ready, kSoftWarps);
+    mbar_init(st_used, kSoftWarps);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (ntiles > 0) {
+    if (warp == 0 && lane == 0) {
+      // ---------------------------------------------------------- TMA producer
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmG);
+      TileWalker it(a, tb, te, T);
+      uint32_t e = 0;
+      bool ok = true;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        if (li > 0) ok = mbar_wait(k_empty, (li - 1) & 1, abort_flag, a.ws, 0x801);
+        if (!ok) break;
+        mbar_arrive_expect_tx(k_full, C::KV_TILE);
+#pragma unroll
+        for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sK + dh * T * 128, &tmK, k_full, 64 * dh, it.h, int(it.tok0));
+        for (int c = 0; c < C::NCH && ok; ++c) {
+#pragma unroll
+          for (int g = 0; g < 2; ++g) {
+            const int s = int(e % C::NQG);
+            if (e >= uint32_t(C::NQG)) ok = mbar_wait(qg_empty(s), ((e / C::NQG) + 1) & 1, abort_flag, a.ws, 0x802);
+            if (!ok) break;
+            mbar_arrive_expect_tx(qg_full(s), C::QG_CHUNK);
+            const int ghead = g ? int(it.b) * a.H + it.h : it.h;  // G copy is [B*H][P][D]
+#pragma unroll
+            for (int dh = 0; dh < D / 64; ++dh)
+              tma_load_3d(sQG + s * C::QG_CHUNK + dh * C::NC * 128, g ? &tmG : &tmQ, qg_full(s), 64 * dh, c * C::NC,
+                          ghead);
+            ++e;
+          }
+          if (c == 0 && ok) {  // V right after the first chunk: dA(0) needs it next
+            if (li > 0) ok = mbar_wait(v_empty, (li - 1) & 1, abort_flag, a.ws, 0x803);
+            if (!ok) break;
+            mbar_arrive_expect_tx(v_full, C::KV_TILE);
+#pragma unroll
+            for (int dh = 0; dh < D / 64; ++dh)
+              tma_load_3d(sV + dh * T * 128, &tmV, v_full, 64 * dh, it.h, int(it.tok0));
+          }
+        }
+        it.next();
+      }
+      if (!ok) {
+        for (uint32_t k = (e > uint32_t(C::NQG) ? e - C::NQG : 0); k < e; ++k)
+          mbar_wait_bounded(qg_full(int(k % C::NQG)), (k / C::NQG) & 1, 200000000ull);
+        mbar_wait_bounded(k_full, (ntiles - 1) & 1, 200000000ull);
+        mbar_wait_bounded(v_full, (ntiles - 1) & 1, 200000000ull);
+      }
+    } else if (warp == 1 && lane == 0) {
+      // ---------------------------------------------------------- UMMA issuer
+      constexpr uint32_t idS = idesc_bf16(128, C::NC, 0, 0);  // [tok x chunk], K = d
+      constexpr uint32_t idTD = idesc_bf16(128, D, 0, 1);     // [tok x d], K = chunk prototypes
+      bool ok = true;
+      auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
+      };
+      uint32_t g = 0;  // global chunk counter
+      for (int li = 0; li < ntiles && ok; ++li) {
+        wt(k_full, li & 1, 0x901);
+        for (int c = 0; c < C::NCH && ok; ++c, ++g) {
+          const uint32_t eQ = 2 * g, eG = eQ + 1;
+          const int sq = int(eQ % C::NQG), sg = int(eG % C::NQG);
+          const uint32_t aQ = sQG + sq * C::QG_CHUNK, aG = sQG + sg * C::QG_CHUNK;
+          // S_c = K Q_c^T
+          wt(qg_full(sq), (eQ / C::NQG) & 1, 0x902);
+          if (g > 0) wt(sd_free_da, (g - 1) & 1, 0x903);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k)
+            umma_ss(tmem + C::SD_COL, sdesc(sK + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                    sdesc(aQ + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
+          umma_commit(s_full);
+          if (c == C::NCH - 1) umma_commit(k_empty);
+          // dA_c = V G_c^T
+          if (c == 0) wt(v_full, li & 1, 0x904);
+          wt(qg_full(sg), (eG / C::NQG) & 1, 0x905);
+          wt(sd_free_s, g & 1, 0x906);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k)
+            umma_ss(tmem + C::SD_COL, sdesc(sV + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                    sdesc(aG + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
+          umma_commit(da_full);
+          if (c == C::NCH - 1) umma_commit(v_empty);
+          // dV += A G_c, qbar += A Q_c
+          wt(a_full, g & 1, 0x907);
+          if (c == 0 && li > 0) wt(acc_empty, (li - 1) & 1, 0x908);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < C::NC / 16; ++k) {
+            const uint64_t ad = sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024);
+            const uint32_t acc = (c == 0 && k == 0) ? 0u : 1u;
+            umma_ss(tmem + C::DV_COL, ad, sdesc(aG + k * 2048, C::NC * 128, 1024), idTD, acc);
+            umma_ss(tmem + C::QB_COL, ad, sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, acc);
+          }
+          umma_commit(ab_empty);
+          umma_commit(qg_empty(sg));
+          // u += E Q_c
+          wt(e_full, g & 1, 0x909);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < C::NC / 16; ++k)
+            umma_ss(tmem + C::U_COL, sdesc(sEB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                    sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, (c == 0 && k == 0) ? 0u : 1u);
+          umma_commit(eb_empty);
+          umma_commit(qg_empty(sq));
+          if (c == C::NCH - 1) umma_commit(acc_full);
+        }
+      }
+      umma_commit(drain);
+      mbar_wait_bounded(drain, 0, 200000000ull);
+    } else if (warp >= kSoftWarp0) {
+      // ------------------------------------------------ softmax + epilogue
+      const int sw = (warp - kSoftWarp0) >> 2, q = warp & 3, row = 32 * q + lane;
+      const uint32_t lane_off = uint32_t(32 * q) << 16;
+      const float c2 = a.scale * 1.4426950408889634f;
+      float* stats = reinterpret_cast<float*>(smem + C::OFF_STATS);
+      TileWalker cur(a, tb, te, T);
+      bool ok = true;
+      auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
+      };
+      uint32_t g = 0;
+      auto put_tile = [&](uint8_t* base, const uint32_t* pk) {
+        uint8_t* rowp = base + row * 128;
+#pragma unroll
+        for (int k = 0; k < C::HALF / 8; ++k) {
+          const int p = sw * C::HALF + 8 * k;
+          const int blk = p >> 6, chunk = (p & 63) >> 3;
+          *reinterpret_cast<uint4*>(rowp + blk * (T * 128) + ((chunk ^ (row & 7)) << 4)) =
+              make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+        }
+      };
+      for (int li = 0; li < ntiles && ok; ++li) {
+        const bool valid = row < cur.n;
+        const int64_t tok = cur.tok0 + row;
+        const float L2 = valid ? lse[tok * a.H + cur.h] * 1.4426950408889634f : 0.f;
+        float Dp = 0.f;
+        for (int c = 0; c < C::NCH && ok; ++c, ++g) {
+          uint32_t apk[C::HALF / 2];
+          float v[32];
+          ok = wwait(s_full, g & 1, 0xA01);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int cc = 0; cc < C::HALF / 32; ++cc) {
+            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * cc, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float x0 = valid ? ex2(fmaf(v[2 * j], c2, -L2)) : 0.f;
+              const float x1 = valid ? ex2(fmaf(v[2 * j + 1], c2, -L2)) : 0.f;
+              apk[16 * cc + j] = pack_bf16(x0, x1);
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sd_free_s);
+          if (g > 0) {
+            ok = wwait(ab_empty, (g - 1) & 1, 0xA02);
+            if (!ok) break;
+          }
+          put_tile(smem + C::OFF_AB, apk);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(a_full);
+          // E = A o dA
+          ok = wwait(da_full, g & 1, 0xA03);
+          if (!ok) break;
+          tc_fence_after();
+          uint32_t epk[C::HALF / 2];
+#pragma unroll
+          for (int cc = 0; cc < C::HALF / 32; ++cc) {
+            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * cc, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const uint32_t w = apk[16 * cc + j];
+              const float e0 = bf16lo(w) * v[2 * j], e1 = bf16hi(w) * v[2 * j + 1];
+              Dp += e0 + e1;
+              epk[16 * cc + j] = pack_bf16(e0, e1);
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sd_free_da);
+          if (g > 0) {
+            ok = wwait(eb_empty, (g - 1) & 1, 0xA04);
+            if (!ok) break;
+          }
+          put_tile(smem + C::OFF_EB, epk);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(e_full);
+        }
+        if (!ok) break;
+        // D_i = (half from warpgroup 0) + (half from warpgroup 1), same order in both
+        if (li > 0) {
+          ok = wwait(st_used, (li - 1) & 1, 0xA05);
+          if (!ok) break;
+        }
+        stats[sw * T + row] = Dp;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(st_ready);
+        ok = wwait(st_ready, li & 1, 0xA06);
+        if (!ok) break;
+        const float Dv = stats[row] + stats[T + row];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(st_used);
+        if (sw == 0 && valid) Dco[tok * a.H + cur.h] = Dv;
+        // epilogue: dV and dK = scale (u - D qbar) for this warpgroup's column half
+        ok = wwait(acc_full, li & 1, 0xA07);
+        if (!ok) break;
+        tc_fence_after();
+        {
+          __nv_bfloat16* dvr = dV + (tok * a.H + cur.h) * int64_t(D) + sw * (D / 2);
+          store_row_bf16<D / 2>(tmem + lane_off + C::DV_COL + sw * (D / 2), dvr, 1.f, valid);
+          __nv_bfloat16* dkr = dK + (tok * a.H + cur.h) * int64_t(D) + sw * (D / 2);
+          float uu[32], qb[32];
+#pragma unroll
+          for (int cc = 0; cc < D / 2; cc += 32) {
+            tmem_ld32(tmem + lane_off + C::U_COL + sw * (D / 2) + cc, uu);
+            tmem_ld32(tmem + lane_off + C::QB_COL + sw * (D / 2) + cc, qb);
+            tmem_ld_wait();
+            if (valid) {
+              uint4* o = reinterpret_cast<uint4*>(dkr + cc);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                float x[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) x[j] = a.scale * fmaf(-Dv, qb[8 * k + j], uu[8 * k + j]);
+                o[k] = make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]),
+                                  pack_bf16(x[6], x[7]));
+              }
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty);
+        cur.next();
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+}  // namespace tcb
+}  // namespace sa
+
+namespace sa {
+namespace tcb {
+
+// dsketch fp32 -> bf16 copy in the workspace, the layout TMA streams ([B*H][P][D])
+__global__ void to_bf16_kernel(const float* __restrict__ src, __nv_bfloat16* __restrict__ dst, int64_t n8,
+                               const void* ws) {
+  if (ws_failed(ws)) return;
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n8; i += int64_t(gridDim.x) * blockDim.x) {
+    const float4 x = reinterpret_cast<const float4*>(src)[2 * i];
+    const float4 y = reinterpret_cast<const float4*>(src)[2 * i + 1];
+    reinterpret_cast<uint4*>(dst)[i] =
+        make_uint4(pack_bf16(x.x, x.y), pack_bf16(x.z, x.w), pack_bf16(y.x, y.y), pack_bf16(y.z, y.w));
+  }
+}
+
+template <int D, int P>
+static cudaError_t launch_tok_t(const Args& a, int W, const __nv_bfloat16* gbf, const float* lse, float* Dco,
+                                void* dK, void* dV, cudaStream_t st) {
+  using C = TokCfg<D, P>;
+  CUtensorMap tk, tv, tq, tg;
+  if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
+      !make_q_map(&tq, a.Q, a.H, a.P, D, C::NC) || !make_q_map(&tg, gbf, a.B * a.H, a.P, D, C::NC))
+    return cudaErrorInvalidValue;
+  auto fn = &tc_bwd_tok_kernel<D, P>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  fn<<<W, kThreads, C::SMEM, st>>>(tk, tv, tq, tg, a, lse, Dco, static_cast<__nv_bfloat16*>(dK),
+                                   static_cast<__nv_bfloat16*>(dV));
+  return cudaGetLastError();
+}
+
+}  // namespace tcb
+
+bool tc_bwd_split(int P, int d) { return d == 128 && (P == 256 || P == 512); }
+
+cudaError_t launch_tc_g_bf16(const Args& a, const float* dsk, __nv_bfloat16* gbf, cudaStream_t st) {
+  const int64_t n8 = int64_t(a.B) * a.H * a.P * a.d / 8;
+  tcb::to_bf16_kernel<<<1024, 256, 0, st>>>(dsk, gbf, n8, a.ws);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tc_bwd_tok(const Args& a, int W, const float* dsk, __nv_bfloat16* gbf, const float* lse,
+                              float* Dco, void* dK, void* dV, cudaStream_t st) {
+  (void)dsk;
+  if (a.N == 0) return cudaSuccess;
+  if (a.P == 512) return tcb::launch_tok_t<128, 512>(a, W, gbf, lse, Dco, dK, dV, st);
+  return tcb::launch_tok_t<128, 256>(a, W, gbf, lse, Dco, dK, dV, st);
+}
+
+cudaError_t launch_tc_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
+                             cudaStream_t st) {
+  if (a.N == 0) return cudaSuccess;
+  return tcb::launch_bwd_t<128, 128, tcb::kSlice>(a, W, dsk, lse, Dco, nullptr, nullptr, st);
+}
+
+int tc_bwd_dq_workers(int num_sms, int P) {
+  const int w = num_sms / (P / 128);
+  return w < 1 ? 1 : w;
 }
 
 }  // namespace sa
