@@ -249,25 +249,28 @@ def run_ours(args, spec, lens):
     bw = rf.bwd_work(tokens, B, H, P, d, eb, lse_in=True)
     peak_t = pk["bf16_tflops_sustained"]
 
-    def roof(work, kms, kn, name):
+    def roof(work, kms, kn, name, calls):
+        """Achieved rate of a call's main kernels: algorithmic work of one call
+        divided by the summed device time of its main-kernel launches."""
         if kn == 0:
             return None
-        avg_s = kms / kn / 1e3
+        per_call_s = kms / calls / 1e3
         t_tensor = work.flops / (peak_t * 1e12)
         t_hbm = work.bytes / (pk["hbm_gbs"] * 1e9)
         if t_tensor >= t_hbm:
-            ach, peak, unit, bound = work.flops / avg_s / 1e12, peak_t, "TFLOP/s", "tensor"
+            ach, peak, unit, bound = work.flops / per_call_s / 1e12, peak_t, "TFLOP/s", "tensor"
         else:
-            ach, peak, unit, bound = work.bytes / avg_s / 1e9, pk["hbm_gbs"], "GB/s", "hbm"
+            ach, peak, unit, bound = work.bytes / per_call_s / 1e9, pk["hbm_gbs"], "GB/s", "hbm"
         return {"kernel": name, "bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
                 "traffic": traffic_for(name), "avg_launch_ms": kms / kn, "launches": kn,
+                "launches_per_call": kn // calls, "ms_per_call": kms / calls,
                 "peak_source": f"{pk['source']} ({'bf16 sustained' if unit == 'TFLOP/s' else 'HBM copy'})",
-                "algorithmic_per_launch": work.flops if unit == "TFLOP/s" else work.bytes}
+                "algorithmic_per_call": work.flops if unit == "TFLOP/s" else work.bytes}
 
     bwd_name = binding.sa_main_kernel_name(P, d, binding.SA_BF16, True)
     fwd_name = binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
-    r_bwd = roof(bw, bwd_k_ms, bwd_k_n, bwd_name)
-    r_fwd = roof(fw, fwd_k_ms, fwd_k_n, fwd_name)
+    r_bwd = roof(bw, bwd_k_ms, bwd_k_n, bwd_name, args.steps)
+    r_fwd = roof(fw, fwd_k_ms, fwd_k_n, fwd_name, args.steps)
     step_w = rf.step_work(tokens, B, H, P, d, eb)
     t_roof = rf.roofline_time(step_w, peak_t, pk["hbm_gbs"])
 
