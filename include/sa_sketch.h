@@ -93,6 +93,29 @@ sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens,
                         void* dV, float* dQ, void* workspace, size_t ws_bytes,
                         void* stream);
 
+/* Allocation-free forward (the paper has no counterpart; this is a library
+ * convenience).  For callers that cannot provide a workspace: for example a
+ * plugin or custom-operator hook that receives only its input and output
+ * buffers and may not allocate device memory, or a service running inside a
+ * device-memory budget fixed in advance.  Same arguments and results as
+ * sa_sketch_fwd without the workspace: the scratch comes from one fixed array
+ * of sa_noalloc_scratch_bytes() bytes (32 MiB) that this library keeps in
+ * device memory on every GPU where it is loaded, until the process exits.
+ *   - Returns SA_ERR_WORKSPACE, before launching anything, when the call would
+ *     need more scratch than that (large N, B, P or d); use sa_sketch_fwd then.
+ *   - It allocates nothing.  The first call on a device looks up the array's
+ *     device address (cudaGetSymbolAddress, with that device current) and
+ *     caches it; make that first call before any stream capture.
+ *   - All calls share the one array: two calls whose work overlaps on the GPU
+ *     (different streams, or different host threads) race and may corrupt each
+ *     other's results; serialise them.  Each call rewrites everything it reads. */
+sa_status sa_sketch_fwd_noalloc(const void* K, const void* V, const int32_t* cu_seqlens, int B,
+                                int64_t N, const void* Q, int H, int P, int d, float scale,
+                                sa_dtype dt, float* sketch, float* lse, void* stream);
+
+/* Size in bytes of the fixed scratch array used by sa_sketch_fwd_noalloc. */
+size_t sa_noalloc_scratch_bytes(void);
+
 /* Synchronises `stream` and returns the device-detected status of the last call
  * that used this workspace (SA_OK, SA_ERR_BAD_SEQLENS or SA_ERR_TIMEOUT), or
  * SA_ERR_CUDA if the stream itself reports an error. */

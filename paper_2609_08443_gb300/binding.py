@@ -61,6 +61,10 @@ def load() -> ctypes.CDLL:
     lib.sa_main_kernel_name.restype = ctypes.c_char_p
     lib.sa_select_path.argtypes = [i32]
     lib.sa_select_path.restype = i32
+    lib.sa_sketch_fwd_noalloc.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp]
+    lib.sa_sketch_fwd_noalloc.restype = i32
+    lib.sa_noalloc_scratch_bytes.argtypes = []
+    lib.sa_noalloc_scratch_bytes.restype = sz
     lib.sa_plan_host.argtypes = [vp, i32, i32, i32, i32, vp]
     lib.sa_plan_host.restype = i32
     _lib = lib
@@ -207,6 +211,30 @@ def sa_sketch_bwd(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q:
                            _stream(K.device))
     _check(st, "sa_sketch_bwd")
     return dK, dV, dQ
+
+
+def sa_sketch_fwd_noalloc(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
+                          scale: Optional[float] = None, out: Optional[torch.Tensor] = None,
+                          lse_out: Optional[torch.Tensor] = None):
+    """Forward without a workspace: for callers that may not allocate device
+    memory when they run this (the library's fixed scratch array is used; see
+    include/sa_sketch.h).  ``out`` and ``lse_out`` are the caller's buffers;
+    when they are not given they are created here, before the call."""
+    lib = load()
+    _validate(K, V, cu_seqlens, Q)
+    N, H, d = K.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    sketch = out if out is not None else torch.empty((B, H, P, d), dtype=torch.float32, device=K.device)
+    st = lib.sa_sketch_fwd_noalloc(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, _dt(K),
+                                   _ptr(sketch), _ptr(lse_out), _stream(K.device))
+    _check(st, "sa_sketch_fwd_noalloc")
+    return sketch
+
+
+def sa_noalloc_scratch_bytes() -> int:
+    return int(load().sa_noalloc_scratch_bytes())
 
 
 def sa_plan_host(cu_seqlens_host, H: int, tile: int, n_workers: int):
