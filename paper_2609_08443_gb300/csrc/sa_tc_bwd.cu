@@ -47,10 +47,11 @@ struct BCfg {
   static constexpr int NBAR = 2 * NSLOT + 20;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int SMEM = OFF_MISC + 16;
+  static constexpr int NSD = (MODE == kSlice) ? 2 : 1;  // S/dA buffers (slice mode has TMEM to spare)
   static constexpr int SD_COL = 0;
   static constexpr int DV_COL = PS;
   static constexpr int DK_COL = PS + D;
-  static constexpr int DQ_COL = (MODE == kFull) ? PS + 2 * D : PS;
+  static constexpr int DQ_COL = (MODE == kFull) ? PS + 2 * D : NSD * PS;
   static constexpr int TMEM_COLS = tmem_cols_for(DQ_COL + (PS / 128) * D);
   static constexpr int HALF = PS / 2;
   static_assert(TMEM_COLS <= 512, "TMEM budget");
@@ -200,20 +201,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
       };
-      // S(i) = K(i) Q^T into the S/dA columns
-      auto issue_S = [&](uint32_t kslot) {
+      auto sdcol = [&](int i) { return uint32_t(C::SD_COL + (i % C::NSD) * PS); };
+      // S(i) = K(i) Q^T into an S/dA buffer
+      auto issue_S = [&](uint32_t kslot, uint32_t col) {
         const uint32_t kaddr = sRing + kslot * C::KV_TILE;
 #pragma unroll
         for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + C::SD_COL, sdesc(kaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+          umma_ss(tmem + col, sdesc(kaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
                   sdesc(sQ + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
       };
+      TileWalker nx2(a, tb, te, T);
+      nx2.next();
+      nx2.next();
       wt(q_full, 0, 0x501);
       wt(ring_full(0), 0, 0x502);
       if (ok) {
         tc_fence_after();
-        issue_S(0);
+        issue_S(0, sdcol(0));
         umma_commit(s_full);
+        // slice mode: Q is read only by S, so it may be replaced after the last S of a head
+        if (MODE == kSlice && (ntiles == 1 || nxt.h != cur.h)) umma_commit(q_empty);
       }
       bool first_of_hp = true;
       for (int li = 0; li < ntiles && ok; ++li) {
@@ -232,7 +239,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t vaddr = sRing + sV * C::KV_TILE;
 #pragma unroll
           for (int k = 0; k < D / 16; ++k)
-            umma_ss(tmem + C::SD_COL, sdesc(vaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+            umma_ss(tmem + sdcol(li), sdesc(vaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
                     sdesc(sG + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
         }
         umma_commit(da_full);
@@ -251,21 +258,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
         if (cur.seg_last) umma_commit(g_empty);
-        // ---- S(i+1), early when the head (and so Q) stays the same
         const bool more = li + 1 < ntiles;
-        const bool hoist = more && nxt.h == cur.h;
-        if (hoist) {
-          wt(sd_free_da, li & 1, 0x508);
-          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0x509);
+        const bool newhead = more && nxt.h != cur.h;
+        // ---- S(i+1) before dK/dQ(i) when its buffer and Q allow it
+        const bool early = more && (C::NSD == 2 || !newhead);
+        if (early) {
+          if (C::NSD == 2) {
+            if (newhead) {
+              ++hc;
+              wt(q_full, hc & 1, 0x508);
+            }
+            if (li >= 1) wt(sd_free_da, (li - 1) & 1, 0x509);
+          } else {
+            wt(sd_free_da, li & 1, 0x509);
+          }
+          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0x50A);
           if (!ok) break;
           tc_fence_after();
-          issue_S((eK + 2) % C::NSLOT);
+          issue_S((eK + 2) % C::NSLOT, sdcol(li + 1));
           umma_commit(s_full);
+          if (MODE == kSlice && (li + 2 >= ntiles || nx2.h != nxt.h)) umma_commit(q_empty);
         }
         // ---- dK(i) = dS Q, dQ += dS^T K
-        wt(ds_full, li & 1, 0x50A);
-        if (MODE == kFull && li > 0) wt(dk_empty, (li - 1) & 1, 0x50B);
-        if (first_of_hp && hp > 0) wt(dq_empty, (hp - 1) & 1, 0x50C);
+        wt(ds_full, li & 1, 0x50B);
+        if (MODE == kFull && li > 0) wt(dk_empty, (li - 1) & 1, 0x50C);
+        if (first_of_hp && hp > 0) wt(dq_empty, (hp - 1) & 1, 0x50D);
         if (!ok) break;
         tc_fence_after();
         if (MODE == kFull) {
@@ -285,26 +302,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         umma_commit(ab_empty);
         umma_commit(ring_empty(sK));
-        const bool last_of_hp = !more || nxt.h != cur.h;
+        const bool last_of_hp = !more || newhead;
         if (last_of_hp) {
           umma_commit(dq_full);
-          umma_commit(q_empty);
+          if (MODE == kFull) umma_commit(q_empty);  // dK read Q up to here
           ++hp;
         }
         first_of_hp = last_of_hp;
-        // ---- S(i+1) after a head change (Q replaced once dK(i) is done)
-        if (more && !hoist) {
+        // ---- S(i+1) after a head change in full mode (Q replaced once dK(i) is done)
+        if (more && !early) {
           ++hc;
-          wt(q_full, hc & 1, 0x50D);
-          wt(sd_free_da, li & 1, 0x50E);
-          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0x50F);
+          wt(q_full, hc & 1, 0x50E);
+          wt(sd_free_da, li & 1, 0x50F);
+          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0x510);
           if (!ok) break;
           tc_fence_after();
-          issue_S((eK + 2) % C::NSLOT);
+          issue_S((eK + 2) % C::NSLOT, sdcol(li + 1));
           umma_commit(s_full);
         }
         cur.next();
         nxt.next();
+        nx2.next();
       }
       umma_commit(drain);
       mbar_wait_bounded(drain, 0, 200000000ull);
@@ -369,21 +387,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       };
       uint32_t apk[C::HALF / 2];  // this thread's A values, bf16 pairs
+      // per-token lse (and D_i in slice mode), loaded one tile ahead
+      float lse_cur = row < cur.n ? lse[(cur.tok0 + row) * a.H + cur.h] : 0.f;
+      float d_cur = (MODE == kSlice && row < cur.n) ? Dco_in[(cur.tok0 + row) * a.H + cur.h] : 0.f;
       for (int li = 0; li < ntiles && ok; ++li) {
         const bool valid = row < cur.n;
         const int64_t tok = cur.tok0 + row;
         const uint32_t eV = 2u * li + 1;
         const int sV = int(eV % C::NSLOT);
+        const uint32_t sdc = C::SD_COL + (li % C::NSD) * PS;
+        float lse_nxt, d_nxt = 0.f;
+        {
+          int64_t t0n;
+          int nn, hn;
+          cur.peek_next(t0n, nn, hn);
+          lse_nxt = row < nn ? lse[(t0n + row) * a.H + hn] : 0.f;
+          if (MODE == kSlice) d_nxt = row < nn ? Dco_in[(t0n + row) * a.H + hn] : 0.f;
+        }
         // ---- A = exp(scale S - lse)
         ok = wwait(s_full, li & 1, 0x701);
         if (!ok) break;
         tc_fence_after();
         {
-          const float L2 = valid ? lse[tok * a.H + cur.h] * 1.4426950408889634f : 0.f;
+          const float L2 = lse_cur * 1.4426950408889634f;
           float v[32];
 #pragma unroll
           for (int c = 0; c < C::HALF / 32; ++c) {
-            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * c, v);
+            tmem_ld32(tmem + lane_off + sdc + sw * C::HALF + 32 * c, v);
             tmem_ld_wait();
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
@@ -457,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive(ring_empty(sV));
           }
         } else {
-          Dv = valid ? Dco_in[tok * a.H + cur.h] : 0.f;
+          Dv = d_cur;
         }
         // ---- dS = A o (dA - D) -> shared memory (over A, whose readers are done)
         ok = wwait(da_full, li & 1, 0x704);
@@ -468,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           float v[32];
 #pragma unroll
           for (int c = 0; c < C::HALF / 32; ++c) {
-            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * c, v);
+            tmem_ld32(tmem + lane_off + sdc + sw * C::HALF + 32 * c, v);
             tmem_ld_wait();
             uint32_t o[16];
 #pragma unroll
@@ -492,6 +522,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive(sd_free_da);
           mbar_arrive(ds_full);
         }
+        lse_cur = lse_nxt;
+        d_cur = d_nxt;
         cur.next();
       }
       if (ok) {
@@ -795,10 +827,17 @@ __global__ void __launch_bounds__(kThreads, 1)
               make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
         }
       };
+      float lse_cur = row < cur.n ? lse[(cur.tok0 + row) * a.H + cur.h] : 0.f;
       for (int li = 0; li < ntiles && ok; ++li) {
         const bool valid = row < cur.n;
         const int64_t tok = cur.tok0 + row;
-        const float L2 = valid ? lse[tok * a.H + cur.h] * 1.4426950408889634f : 0.f;
+        const float L2 = lse_cur * 1.4426950408889634f;
+        {
+          int64_t t0n;
+          int nn, hn;
+          cur.peek_next(t0n, nn, hn);
+          lse_cur = row < nn ? lse[(t0n + row) * a.H + hn] : 0.f;
+        }
         float Dp = 0.f;
         for (int c = 0; c < C::NCH && ok; ++c, ++g) {
           uint32_t apk[C::HALF / 2];

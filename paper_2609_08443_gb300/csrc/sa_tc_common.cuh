@@ -54,6 +54,27 @@ struct TileWalker {
     seg_first = (k == 0) || (t == tb);
     seg_last = (k == nk - 1) || (t == te - 1);
   }
+  // First token, size and head of the tile after this one (n = 0 past the range).
+  __device__ void peek_next(int64_t& tok0_n, int& n_n, int& h_n) const {
+    if (t + 1 >= te) {
+      tok0_n = 0;
+      n_n = 0;
+      h_n = h;
+      return;
+    }
+    if (k + 1 < nk) {
+      const int64_t L = int64_t(cu[b + 1]) - int64_t(cu[b]);
+      tok0_n = tok0 + Tt;
+      const int64_t left = L - (k + 1) * Tt;
+      n_n = int(left < Tt ? left : Tt);
+      h_n = h;
+    } else {
+      const TileRef r = locate_tile(t + 1, tph, prefix, cu, B, Tt);
+      tok0_n = r.tok0;
+      n_n = r.n;
+      h_n = r.h;
+    }
+  }
   __device__ void next() {
     ++t;
     if (t >= te) return;

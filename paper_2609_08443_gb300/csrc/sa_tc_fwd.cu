@@ -266,11 +266,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       TileWalker cur(a, tb, te, T);
       int seg_idx = 0;
       bool ok = true;
+      // sliced mode: this token's lse, loaded one tile ahead
+      float lse_cur = (MODE == kSliced && row < cur.n) ? lse_in[(cur.tok0 + row) * a.H + cur.h] : 0.f;
       // every wait result is made warp-uniform so a timeout never splits a warp
       auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
       };
       for (int li = 0; li < ntiles && ok; ++li) {
+        float lse_nxt = 0.f;
+        if (MODE == kSliced) {  // next tile's lse, issued before this tile's scores are live
+          int64_t t0n;
+          int nn, hn;
+          cur.peek_next(t0n, nn, hn);
+          lse_nxt = row < nn ? lse_in[(t0n + row) * a.H + hn] : 0.f;
+        }
         ok = wwait(s_full, li & 1, 0x301);
         if (!ok) break;
         tc_fence_after();
@@ -315,7 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = 0; j < C::HALF; ++j) v[j] *= f;
           if (sw == 0 && valid && lse_out) lse_out[tok * a.H + cur.h] = M * a.scale + logf(Z);
         } else {
-          const float L2 = valid ? lse_in[tok * a.H + cur.h] * 1.4426950408889634f : 0.f;
+          const float L2 = lse_cur * 1.4426950408889634f;
 #pragma unroll
           for (int j = 0; j < C::HALF; ++j) v[j] = ex2(fmaf(v[j], c2, -L2));
         }
@@ -343,6 +352,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(w_full);
+        lse_cur = lse_nxt;
         if (cur.seg_last) {
           ok = wwait(o_full, seg_idx & 1, 0x303);
           if (!ok) break;
