@@ -1005,14 +1005,373 @@ cudaError_t launch_tc_bwd_tok(const Args& a, int W, const float* dsk, __nv_bfloa
 }
 
 cudaError_t launch_tc_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
-                             cudaStream_t st) {
-  if (a.N == 0) return cudaSuccess;
-  return tcb::launch_bwd_t<128, 128, tcb::kSlice>(a, W, dsk, lse, Dco, nullptr, nullptr, st);
-}
+                             cudaStream_t st);
 
 int tc_bwd_dq_workers(int num_sms, int P) {
   const int w = num_sms / (P / 128);
   return w < 1 ? 1 : w;
 }
 
+}  // namespace sa
+
+// ================================================================ dQ (slices)
+// Prototype side of the backward: one slice of PS = 128 prototypes per CTA,
+// prototypes on TMEM lanes, tokens on columns:
+//   S  = Q_r K^T,  dA = G_r V^T                (UMMA, [PS x 128 tokens])
+//   dS = exp(scale S - lse_t) o (dA - D_t)     (registers; lse_t and D_t are
+//                                               per-column values, no reduction)
+//   dQ_r += dS K                               (UMMA with dS as the A operand
+//                                               straight from TMEM)
+// D_t comes from the token-side kernel.  Keeping dS in TMEM spares the
+// shared-memory round trip that bounds the other kernels.
+namespace sa {
+namespace tcb {
+
+template <int D, int PS>
+struct QCfg {
+  static constexpr int KV_TILE = T * D * 2;
+  static constexpr int QB = PS * D * 2;
+  static constexpr int NSLOT = 4;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_G = QB;
+  static constexpr int OFF_RING = 2 * QB;
+  static constexpr int OFF_COL = OFF_RING + NSLOT * KV_TILE;  // [2 bufs][lse2 | D][128] fp32
+  static constexpr int OFF_BAR = OFF_COL + 2 * 2 * T * 4;
+  static constexpr int NBAR = 2 * NSLOT + 20;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+  static constexpr int SMEM = OFF_MISC + 16;
+  static constexpr int S_COL = 0, DA_COL = T, DS_COL = 2 * T, DQ_COL = 2 * T + T / 2;
+  static constexpr int TMEM_COLS = tmem_cols_for(DQ_COL + D);
+  static_assert(PS == 128 && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
+};
+
+template <int D, int PS>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                     const __grid_constant__ CUtensorMap tmQ, Args a, const float* __restrict__ dsk,
+                     const float* __restrict__ lse, const float* __restrict__ Dco) {
+  using C = QCfg<D, PS>;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (ws_failed(a.ws)) return;
+  if (smem_u32(smem) & 1023u) {
+    if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xB31u);
+    return;
+  }
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t sQ = sbase + C::OFF_Q, sG = sbase + C::OFF_G, sRing = sbase + C::OFF_RING;
+  const uint32_t bar0 = sbase + C::OFF_BAR;
+  auto ring_full = [&](int s) { return bar0 + 8u * s; };
+  auto ring_empty = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
+  const uint32_t b1 = bar0 + 8u * (2 * C::NSLOT);
+  const uint32_t q_full = b1, q_empty = b1 + 8, g_full = b1 + 16, g_empty = b1 + 24, s_full = b1 + 32,
+                 s_free = b1 + 40, da_full = b1 + 48, da_free = b1 + 56, ds_full = b1 + 64, ds_empty = b1 + 72,
+                 dq_empty = b1 + 80, col_full0 = b1 + 88, col_empty0 = b1 + 104, drain = b1 + 120;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+  float* cols = reinterpret_cast<float*>(smem + C::OFF_COL);
+  const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
+  const int64_t total = tph * a.H;
+  const int W = gridDim.x, wk = blockIdx.x, slice = blockIdx.y;
+  const int p0 = slice * PS;
+  const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
+  const int ntiles = int(te - tb);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(ring_full(s), 1);
+      mbar_init(ring_empty(s), 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    mbar_init(g_full, 2);
+    mbar_init(g_empty, 1);
+    mbar_init(s_full, 1);
+    mbar_init(s_free, kSoftWarps);
+    mbar_init(da_full, 1);
+    mbar_init(da_free, kSoftWarps);
+    mbar_init(ds_full, kSoftWarps);
+    mbar_init(ds_empty, 1);
+    mbar_init(dq_empty, kSoftWarps);
+    mbar_init(col_full0, 2);
+    mbar_init(col_full0 + 8, 2);
+    mbar_init(col_empty0, kSoftWarps);
+    mbar_init(col_empty0 + 8, kSoftWarps);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (ntiles > 0) {
+    if (warp == 0 && lane == 0) {
+      // ---------------------------------------------------------- TMA producer
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      tma_prefetch_desc(&tmQ);
+      TileWalker it(a, tb, te, T);
+      int hc = 0, prev_h = -1;
+      uint32_t e = 0;
+      bool ok = true;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        if (it.h != prev_h) {
+          if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0xC01);
+          if (!ok) break;
+          mbar_arrive_expect_tx(q_full, C::QB);
+#pragma unroll
+          for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.h);
+          prev_h = it.h;
+          ++hc;
+        }
+#pragma unroll
+        for (int kv = 0; kv < 2; ++kv) {
+          const int s = int(e % C::NSLOT);
+          if (e >= uint32_t(C::NSLOT)) ok = mbar_wait(ring_empty(s), ((e / C::NSLOT) + 1) & 1, abort_flag, a.ws, 0xC02);
+          if (!ok) break;
+          mbar_arrive_expect_tx(ring_full(s), C::KV_TILE);
+#pragma unroll
+          for (int dh = 0; dh < D / 64; ++dh)
+            tma_load_3d(sRing + s * C::KV_TILE + dh * T * 128, kv ? &tmV : &tmK, ring_full(s), 64 * dh, it.h,
+                        int(it.tok0));
+          ++e;
+        }
+        it.next();
+      }
+      if (!ok) {
+        for (uint32_t k = (e > uint32_t(C::NSLOT) ? e - C::NSLOT : 0); k < e; ++k)
+          mbar_wait_bounded(ring_full(int(k % C::NSLOT)), (k / C::NSLOT) & 1, 200000000ull);
+      }
+    } else if (warp == 1 && lane == 0) {
+      // ---------------------------------------------------------- UMMA issuer
+      constexpr uint32_t idPT = idesc_bf16(128, T, 0, 0);  // [proto x tok], K = d
+      constexpr uint32_t idQ = idesc_bf16(128, D, 0, 1);   // [proto x d], K = tokens, A from TMEM
+      TileWalker cur(a, tb, te, T), nxt(a, tb, te, T), nx2(a, tb, te, T);
+      nxt.next();
+      nx2.next();
+      nx2.next();
+      int hc = 0, gc = 0, hp = 0;
+      bool ok = true;
+      auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
+      };
+      auto issue_pt = [&](uint32_t dcol, uint32_t aop, uint32_t bop) {  // [proto x tok] = aop bop^T
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          umma_ss(tmem + dcol, sdesc(aop + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024),
+                  sdesc(bop + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024), idPT, k > 0 ? 1u : 0u);
+      };
+      wt(q_full, 0, 0xD01);
+      wt(ring_full(0), 0, 0xD02);
+      if (ok) {
+        tc_fence_after();
+        issue_pt(C::S_COL, sQ, sRing);
+        umma_commit(s_full);
+        if (ntiles == 1 || nxt.h != cur.h) umma_commit(q_empty);
+      }
+      bool first_of_hp = true;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        const uint32_t eK = 2u * li, eV = eK + 1;
+        const int sK = int(eK % C::NSLOT), sV = int(eV % C::NSLOT);
+        // ---- dA(i) = G_r V(i)^T
+        if (cur.seg_first) {
+          wt(g_full, gc & 1, 0xD03);
+          ++gc;
+        }
+        wt(ring_full(sV), (eV / C::NSLOT) & 1, 0xD04);
+        if (li > 0) wt(da_free, (li - 1) & 1, 0xD05);
+        if (!ok) break;
+        tc_fence_after();
+        issue_pt(C::DA_COL, sG, sRing + sV * C::KV_TILE);
+        umma_commit(da_full);
+        umma_commit(ring_empty(sV));
+        if (cur.seg_last) umma_commit(g_empty);
+        // ---- S(i+1) while the softmax warps work on tile i
+        const bool more = li + 1 < ntiles;
+        const bool newhead = more && nxt.h != cur.h;
+        if (more) {
+          if (newhead) {
+            ++hc;
+            wt(q_full, hc & 1, 0xD06);
+          }
+          wt(s_free, li & 1, 0xD07);
+          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0xD08);
+          if (!ok) break;
+          tc_fence_after();
+          issue_pt(C::S_COL, sQ, sRing + ((eK + 2) % C::NSLOT) * C::KV_TILE);
+          umma_commit(s_full);
+          if (li + 2 >= ntiles || nx2.h != nxt.h) umma_commit(q_empty);
+        }
+        // ---- dQ += dS K(i), dS read from TMEM
+        wt(ds_full, li & 1, 0xD09);
+        if (first_of_hp && hp > 0) wt(dq_empty, (hp - 1) & 1, 0xD0A);
+        if (!ok) break;
+        tc_fence_after();
+        {
+          const uint32_t kaddr = sRing + sK * C::KV_TILE;
+#pragma unroll
+          for (int k = 0; k < T / 16; ++k)
+            umma_ts(tmem + C::DQ_COL, tmem + C::DS_COL + 8 * k, sdesc(kaddr + k * 2048, T * 128, 1024), idQ,
+                    (first_of_hp && k == 0) ? 0u : 1u);
+        }
+        umma_commit(ds_empty);
+        umma_commit(ring_empty(sK));
+        const bool last_of_hp = !more || newhead;
+        if (last_of_hp) ++hp;
+        first_of_hp = last_of_hp;
+        cur.next();
+        nxt.next();
+        nx2.next();
+      }
+      umma_commit(drain);
+      mbar_wait_bounded(drain, 0, 200000000ull);
+    } else if (warp == 2 || warp == 3) {
+      // ------------------- dsketch slice (fp32 -> bf16, swizzled) and per-token columns
+      const int t64 = threadIdx.x - 64;
+      TileWalker cur(a, tb, te, T);
+      int gc = 0;
+      bool ok = true;
+      auto hw = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
+      };
+      for (int li = 0; li < ntiles && ok; ++li) {
+        if (cur.seg_first) {
+          if (gc > 0) ok = hw(g_empty, (gc - 1) & 1, 0xE01);
+          if (!ok) break;
+          const float* src = dsk + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D;
+          constexpr int CHUNKS = PS * D / 8;
+          for (int c = t64; c < CHUNKS; c += 64) {
+            const int p = c / (D / 8), dd = (c % (D / 8)) * 8;
+            const float4 x = *reinterpret_cast<const float4*>(src + int64_t(p) * D + dd);
+            const float4 y = *reinterpret_cast<const float4*>(src + int64_t(p) * D + dd + 4);
+            const int dh = dd >> 6, chunk = (dd & 63) >> 3;
+            *reinterpret_cast<uint4*>(smem + C::OFF_G + dh * PS * 128 + p * 128 + ((chunk ^ (p & 7)) << 4)) =
+                make_uint4(pack_bf16(x.x, x.y), pack_bf16(x.z, x.w), pack_bf16(y.x, y.y), pack_bf16(y.z, y.w));
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(g_full);
+          ++gc;
+        }
+        const int buf = li & 1;
+        if (li >= 2) ok = hw(col_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xE02);
+        if (!ok) break;
+        float* cl = cols + buf * 2 * T;
+        for (int t = t64; t < T; t += 64) {
+          const bool v = t < cur.n;
+          const int64_t idx = (cur.tok0 + t) * a.H + cur.h;
+          cl[t] = v ? lse[idx] * 1.4426950408889634f : INFINITY;  // exp2(x - inf) = 0 for padding
+          cl[T + t] = v ? Dco[idx] : 0.f;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(col_full0 + 8 * buf);
+        cur.next();
+      }
+    } else if (warp >= kSoftWarp0) {
+      // ------------------------------------------------ dS + dQ epilogue
+      const int sw = (warp - kSoftWarp0) >> 2, q = warp & 3;
+      const uint32_t lane_off = uint32_t(32 * q) << 16;
+      const float c2 = a.scale * 1.4426950408889634f;
+      TileWalker cur(a, tb, te, T);
+      bool ok = true;
+      auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
+      };
+      int hp = 0;
+      for (int li = 0; li < ntiles && ok; ++li) {
+        const int buf = li & 1;
+        ok = wwait(col_full0 + 8 * buf, (li >> 1) & 1, 0xF01);
+        if (ok) ok = wwait(s_full, li & 1, 0xF02);
+        if (ok) ok = wwait(da_full, li & 1, 0xF03);
+        if (ok && li > 0) ok = wwait(ds_empty, (li - 1) & 1, 0xF04);
+        if (!ok) break;
+        tc_fence_after();
+        const float* cl = cols + buf * 2 * T;
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const int col = 64 * sw + 32 * c;
+          float sv[32], dv[32];
+          tmem_ld32(tmem + lane_off + C::S_COL + col, sv);
+          tmem_ld32(tmem + lane_off + C::DA_COL + col, dv);
+          tmem_ld_wait();
+          if (c == 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+              mbar_arrive(s_free);
+              mbar_arrive(da_free);
+            }
+          }
+          uint32_t pk[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int t = col + 2 * j;
+            const float a0 = ex2(fmaf(sv[2 * j], c2, -cl[t]));
+            const float a1 = ex2(fmaf(sv[2 * j + 1], c2, -cl[t + 1]));
+            pk[j] = pack_bf16(a0 * (dv[2 * j] - cl[T + t]), a1 * (dv[2 * j + 1] - cl[T + t + 1]));
+          }
+          tmem_st16(tmem + lane_off + C::DS_COL + col / 2, pk);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(ds_full);
+          mbar_arrive(col_empty0 + 8 * buf);
+        }
+        // dQ partial of this worker and head at the end of its head piece
+        const bool more = li + 1 < ntiles;
+        int64_t t0n;
+        int nn, hn;
+        cur.peek_next(t0n, nn, hn);
+        if (!more || hn != cur.h) {
+          ok = wwait(ds_empty, li & 1, 0xF05);
+          if (!ok) break;
+          tc_fence_after();
+          float* dst = a.dq_partial + ((int64_t(wk) * a.H + cur.h) * a.P + p0) * D;
+          store_sketch_scaled<D, PS, C::DQ_COL>(tmem, lane_off, sw, q, lane, dst, a.scale);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(dq_empty);
+          ++hp;
+        }
+        cur.next();
+      }
+      (void)hp;
+    }
+  }
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int D, int PS>
+static cudaError_t launch_dq_t(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
+                               cudaStream_t st) {
+  using C = QCfg<D, PS>;
+  CUtensorMap tk, tv, tq;
+  if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
+      !make_q_map(&tq, a.Q, a.H, a.P, D, PS))
+    return cudaErrorInvalidValue;
+  auto fn = &tc_bwd_dq_kernel<D, PS>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  dim3 grid(W, a.P / PS);
+  fn<<<grid, kThreads, C::SMEM, st>>>(tk, tv, tq, a, dsk, lse, Dco);
+  return cudaGetLastError();
+}
+
+}  // namespace tcb
+}  // namespace sa
+
+namespace sa {
+cudaError_t launch_tc_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
+                             cudaStream_t st) {
+  if (a.N == 0) return cudaSuccess;
+  return tcb::launch_dq_t<128, 128>(a, W, dsk, lse, Dco, st);
+}
 }  // namespace sa
