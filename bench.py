@@ -233,6 +233,16 @@ def run_ours(args, spec, lens):
     ms = e0.elapsed_time(e1)
     fwd_k_ms, fwd_k_n = binding.sa_timing_read(binding.SA_KERNEL_FWD_MAIN)
     bwd_k_ms, bwd_k_n = binding.sa_timing_read(binding.SA_KERNEL_BWD_MAIN)
+    per_kernel = {}
+    for cls, label in ((binding.SA_KERNEL_FWD_LSE, "fwd_lse"), (binding.SA_KERNEL_FWD_MAIN, "fwd_main"),
+                       (binding.SA_KERNEL_BWD_MAIN, "bwd_main"), (binding.SA_KERNEL_BWD_DQ, "bwd_dq")):
+        kms, kn = binding.sa_timing_read(cls)
+        if kn:
+            per_kernel[label] = {"ms_per_call": kms / args.steps, "launches": kn}
+    # the backward's main kernels: token side plus prototype-side dQ when split
+    if "bwd_dq" in per_kernel:
+        bwd_k_ms += per_kernel["bwd_dq"]["ms_per_call"] * args.steps
+        bwd_k_n += per_kernel["bwd_dq"]["launches"]
     binding.sa_timing_enable(False)
     if binding.sa_get_device_error(ws) != 0:
         raise RuntimeError("device-side error in the timed region")
@@ -288,7 +298,7 @@ def run_ours(args, spec, lens):
                                   "frac": t_roof["time"] * 1e3 / ms_per_step},
                 "roofline": r_bwd, "roofline_fwd": r_fwd,
                 "cpu_baseline": cpu, "e2e": e2e, "clocks": clk.summary(), "gpu_launches": int(launches),
-                "kernels": {"fwd": fwd_name, "bwd": bwd_name}}
+                "kernels": {"fwd": fwd_name, "bwd": bwd_name}, "kernel_ms": per_kernel}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

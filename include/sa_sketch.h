@@ -126,8 +126,16 @@ const char* sa_status_string(sa_status s);
 
 /* ---- measurement hooks (used by bench.py; not needed for normal use) ------- */
 
-/* Kernel classes whose launches can be timed with CUDA events. */
-typedef enum { SA_KERNEL_FWD_MAIN = 0, SA_KERNEL_BWD_MAIN = 1, SA_KERNEL_AUX = 2 } sa_kernel_class;
+/* Kernel classes whose launches can be timed with CUDA events: the forward's
+ * main kernel, the backward's main (token-side) kernel, small helpers, the
+ * per-token lse pass, and the backward's prototype-side dQ kernel. */
+typedef enum {
+  SA_KERNEL_FWD_MAIN = 0,
+  SA_KERNEL_BWD_MAIN = 1,
+  SA_KERNEL_AUX = 2,
+  SA_KERNEL_FWD_LSE = 3,
+  SA_KERNEL_BWD_DQ = 4
+} sa_kernel_class;
 
 /* Turn event timing of the main kernels on (1) or off (0) and clear the record.
  * When on, every main-kernel launch is bracketed by CUDA events recorded on the

@@ -18,7 +18,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libsa_sketch.so")
 
 SA_F32, SA_BF16 = 0, 1
-SA_KERNEL_FWD_MAIN, SA_KERNEL_BWD_MAIN, SA_KERNEL_AUX = 0, 1, 2
+SA_KERNEL_FWD_MAIN, SA_KERNEL_BWD_MAIN, SA_KERNEL_AUX, SA_KERNEL_FWD_LSE, SA_KERNEL_BWD_DQ = 0, 1, 2, 3, 4
 STATUS = {0: "SA_OK", 1: "SA_ERR_INVALID_ARG", 2: "SA_ERR_UNSUPPORTED", 3: "SA_ERR_WORKSPACE",
           4: "SA_ERR_CUDA", 5: "SA_ERR_TIMEOUT", 6: "SA_ERR_BAD_SEQLENS"}
 

@@ -245,7 +245,7 @@ sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens,
     float* l = lse;
     if (sa::tc_fwd_needs_lse_pass_d(P, d)) {
       if (!l) l = a.lse_scratch;
-      SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tc_lse(a, l, st); }));
+      SA_TRY(launch(SA_KERNEL_FWD_LSE, st, [&] { return sa::launch_tc_lse(a, l, st); }));
     }
     SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_tc_fwd(a, plan.W_fwd, sketch, l, st); }));
   } else {
@@ -286,7 +286,7 @@ sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens,
     SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tc_g_bf16(a, dsketch, gbf, st); }));
     SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
                   [&] { return sa::launch_tc_bwd_tok(a, plan.W_bwd, dsketch, gbf, l, Dco, dK, dV, st); }));
-    SA_TRY(launch(SA_KERNEL_BWD_MAIN, st, [&] { return sa::launch_tc_bwd_dq(a, Wq, dsketch, l, Dco, st); }));
+    SA_TRY(launch(SA_KERNEL_BWD_DQ, st, [&] { return sa::launch_tc_bwd_dq(a, Wq, dsketch, l, Dco, st); }));
     SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, Wq, dQ, st); }));
     return SA_OK;
   }
