@@ -611,13 +611,12 @@ struct TokCfg {
   static constexpr int NCH = P / NC;
   static constexpr int KV_TILE = T * D * 2;
   static constexpr int QG_CHUNK = NC * D * 2;
-  static constexpr int NQG = 3;  // ring of Q / G chunks (entries alternate Q, G)
+  static constexpr int NQG = 4;  // ring of Q / G chunks: even slots Q, odd slots G
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = KV_TILE;
   static constexpr int OFF_QG = 2 * KV_TILE;
-  static constexpr int OFF_AB = OFF_QG + NQG * QG_CHUNK;
-  static constexpr int OFF_EB = OFF_AB + T * NC * 2;
-  static constexpr int OFF_STATS = OFF_EB + T * NC * 2;
+  static constexpr int OFF_AB = OFF_QG + NQG * QG_CHUNK;  // A, then E = A o dA, of one chunk
+  static constexpr int OFF_STATS = OFF_AB + T * NC * 2;
   static constexpr int OFF_BAR = OFF_STATS + 2 * T * 4;
   static constexpr int NBAR = 2 * NQG + 20;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
@@ -643,16 +642,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t sK = sbase + C::OFF_K, sV = sbase + C::OFF_V, sQG = sbase + C::OFF_QG, sAB = sbase + C::OFF_AB,
-                 sEB = sbase + C::OFF_EB;
+  const uint32_t sK = sbase + C::OFF_K, sV = sbase + C::OFF_V, sQG = sbase + C::OFF_QG, sAB = sbase + C::OFF_AB;
   const uint32_t bar0 = sbase + C::OFF_BAR;
   auto qg_full = [&](int s) { return bar0 + 8u * s; };
   auto qg_empty = [&](int s) { return bar0 + 8u * (C::NQG + s); };
   const uint32_t b1 = bar0 + 8u * (2 * C::NQG);
   const uint32_t k_full = b1, k_empty = b1 + 8, v_full = b1 + 16, v_empty = b1 + 24, s_full = b1 + 32,
-                 sd_free_s = b1 + 40, da_full = b1 + 48, sd_free_da = b1 + 56, a_full = b1 + 64, ab_empty = b1 + 72,
-                 e_full = b1 + 80, eb_empty = b1 + 88, acc_full = b1 + 96, acc_empty = b1 + 104, st_ready = b1 + 112,
-                 st_used = b1 + 120, drain = b1 + 128;
+                 sd_free_s = b1 + 40, da_full = b1 + 48, sd_free_da = b1 + 56, a_full = b1 + 64,
+                 ab_free_a = b1 + 72, e_full = b1 + 80, ab_free_e = b1 + 88, acc_full = b1 + 96,
+                 acc_empty = b1 + 104, st_ready = b1 + 112, st_used = b1 + 120, drain = b1 + 128;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
   const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
@@ -674,9 +672,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(da_full, 1);
     mbar_init(sd_free_da, kSoftWarps);
     mbar_init(a_full, kSoftWarps);
-    mbar_init(ab_empty, 1);
+    mbar_init(ab_free_a, 1);
     mbar_init(e_full, kSoftWarps);
-    mbar_init(eb_empty, 1);
+    mbar_init(ab_free_e, 1);
     mbar_init(acc_full, 1);
     mbar_init(acc_empty, kSoftWarps);
     mbar_init(st_ready, kSoftWarps);
@@ -721,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                           ghead);
             ++e;
           }
-          if (c == 0 && ok) {  // V right after the first chunk: dA(0) needs it next
+          if (c == 0 && ok) {  // V right after the first chunk: dA of chunk 0 needs it next
             if (li > 0) ok = mbar_wait(v_empty, (li - 1) & 1, abort_flag, a.ws, 0x803);
             if (!ok) break;
             mbar_arrive_expect_tx(v_full, C::KV_TILE);
@@ -740,68 +738,84 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- UMMA issuer
+      // Order per chunk g: dA_g, dV_g + qbar_g, S_{g+1}, u_g.  S of the next chunk
+      // runs while the softmax warps wait to put E_g where A_g was.
       constexpr uint32_t idS = idesc_bf16(128, C::NC, 0, 0);  // [tok x chunk], K = d
       constexpr uint32_t idTD = idesc_bf16(128, D, 0, 1);     // [tok x d], K = chunk prototypes
       bool ok = true;
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
       };
-      uint32_t g = 0;  // global chunk counter
-      for (int li = 0; li < ntiles && ok; ++li) {
-        wt(k_full, li & 1, 0x901);
-        for (int c = 0; c < C::NCH && ok; ++c, ++g) {
-          const uint32_t eQ = 2 * g, eG = eQ + 1;
-          const int sq = int(eQ % C::NQG), sg = int(eG % C::NQG);
-          const uint32_t aQ = sQG + sq * C::QG_CHUNK, aG = sQG + sg * C::QG_CHUNK;
-          // S_c = K Q_c^T
-          wt(qg_full(sq), (eQ / C::NQG) & 1, 0x902);
-          if (g > 0) wt(sd_free_da, (g - 1) & 1, 0x903);
-          if (!ok) break;
-          tc_fence_after();
+      const uint32_t nchunks = uint32_t(ntiles) * C::NCH;
+      auto issue_S = [&](uint32_t g) {
+        const uint32_t sq = (2 * g) % C::NQG;
+        const uint32_t aQ = sQG + sq * C::QG_CHUNK;
 #pragma unroll
-          for (int k = 0; k < D / 16; ++k)
-            umma_ss(tmem + C::SD_COL, sdesc(sK + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(aQ + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
-          umma_commit(s_full);
-          if (c == C::NCH - 1) umma_commit(k_empty);
-          // dA_c = V G_c^T
-          if (c == 0) wt(v_full, li & 1, 0x904);
-          wt(qg_full(sg), (eG / C::NQG) & 1, 0x905);
-          wt(sd_free_s, g & 1, 0x906);
-          if (!ok) break;
-          tc_fence_after();
+        for (int k = 0; k < D / 16; ++k)
+          umma_ss(tmem + C::SD_COL, sdesc(sK + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                  sdesc(aQ + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
+        umma_commit(s_full);
+        if (g % C::NCH == C::NCH - 1) umma_commit(k_empty);  // last S of the tile
+      };
+      // S_0
+      wt(k_full, 0, 0x901);
+      wt(qg_full(0), 0, 0x902);
+      if (ok) {
+        tc_fence_after();
+        issue_S(0);
+      }
+      for (uint32_t g = 0; g < nchunks && ok; ++g) {
+        const uint32_t li = g / C::NCH, c = g % C::NCH;
+        const uint32_t eQ = 2 * g, eG = eQ + 1;
+        const int sq = int(eQ % C::NQG), sg = int(eG % C::NQG);
+        const uint32_t aQ = sQG + sq * C::QG_CHUNK, aG = sQG + sg * C::QG_CHUNK;
+        // ---- dA_g = V G_g^T (into the S/dA columns once S_g was read)
+        if (c == 0) wt(v_full, li & 1, 0x903);
+        wt(qg_full(sg), (eG / C::NQG) & 1, 0x904);
+        wt(sd_free_s, g & 1, 0x905);
+        if (!ok) break;
+        tc_fence_after();
 #pragma unroll
-          for (int k = 0; k < D / 16; ++k)
-            umma_ss(tmem + C::SD_COL, sdesc(sV + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(aG + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
-          umma_commit(da_full);
-          if (c == C::NCH - 1) umma_commit(v_empty);
-          // dV += A G_c, qbar += A Q_c
-          wt(a_full, g & 1, 0x907);
-          if (c == 0 && li > 0) wt(acc_empty, (li - 1) & 1, 0x908);
-          if (!ok) break;
-          tc_fence_after();
+        for (int k = 0; k < D / 16; ++k)
+          umma_ss(tmem + C::SD_COL, sdesc(sV + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                  sdesc(aG + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
+        umma_commit(da_full);
+        if (c == C::NCH - 1) umma_commit(v_empty);
+        // ---- dV += A G_g, qbar += A Q_g
+        wt(a_full, g & 1, 0x906);
+        if (c == 0 && li > 0) wt(acc_empty, (li - 1) & 1, 0x907);
+        if (!ok) break;
+        tc_fence_after();
 #pragma unroll
-          for (int k = 0; k < C::NC / 16; ++k) {
-            const uint64_t ad = sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024);
-            const uint32_t acc = (c == 0 && k == 0) ? 0u : 1u;
-            umma_ss(tmem + C::DV_COL, ad, sdesc(aG + k * 2048, C::NC * 128, 1024), idTD, acc);
-            umma_ss(tmem + C::QB_COL, ad, sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, acc);
-          }
-          umma_commit(ab_empty);
-          umma_commit(qg_empty(sg));
-          // u += E Q_c
-          wt(e_full, g & 1, 0x909);
-          if (!ok) break;
-          tc_fence_after();
-#pragma unroll
-          for (int k = 0; k < C::NC / 16; ++k)
-            umma_ss(tmem + C::U_COL, sdesc(sEB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, (c == 0 && k == 0) ? 0u : 1u);
-          umma_commit(eb_empty);
-          umma_commit(qg_empty(sq));
-          if (c == C::NCH - 1) umma_commit(acc_full);
+        for (int k = 0; k < C::NC / 16; ++k) {
+          const uint64_t ad = sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024);
+          const uint32_t acc = (c == 0 && k == 0) ? 0u : 1u;
+          umma_ss(tmem + C::DV_COL, ad, sdesc(aG + k * 2048, C::NC * 128, 1024), idTD, acc);
+          umma_ss(tmem + C::QB_COL, ad, sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, acc);
         }
+        umma_commit(ab_free_a);
+        umma_commit(qg_empty(sg));
+        // ---- S_{g+1}
+        if (g + 1 < nchunks) {
+          const uint32_t gn = g + 1;
+          if (gn % C::NCH == 0) wt(k_full, (gn / C::NCH) & 1, 0x908);
+          wt(qg_full(int((2 * gn) % C::NQG)), ((2 * gn) / C::NQG) & 1, 0x909);
+          wt(sd_free_da, g & 1, 0x90A);
+          if (!ok) break;
+          tc_fence_after();
+          issue_S(gn);
+        }
+        // ---- u += E Q_g
+        wt(e_full, g & 1, 0x90B);
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int k = 0; k < C::NC / 16; ++k)
+          umma_ss(tmem + C::U_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+                  sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, (c == 0 && k == 0) ? 0u : 1u);
+        umma_commit(ab_free_e);
+        umma_commit(qg_empty(sq));
+        if (c == C::NCH - 1) umma_commit(acc_full);
       }
       umma_commit(drain);
       mbar_wait_bounded(drain, 0, 200000000ull);
@@ -817,8 +831,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
       };
       uint32_t g = 0;
-      auto put_tile = [&](uint8_t* base, const uint32_t* pk) {
-        uint8_t* rowp = base + row * 128;
+      auto put_tile = [&](const uint32_t* pk) {
+        uint8_t* rowp = smem + C::OFF_AB + row * 128;
 #pragma unroll
         for (int k = 0; k < C::HALF / 8; ++k) {
           const int p = sw * C::HALF + 8 * k;
@@ -860,10 +874,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(sd_free_s);
           if (g > 0) {
-            ok = wwait(ab_empty, (g - 1) & 1, 0xA02);
+            ok = wwait(ab_free_e, (g - 1) & 1, 0xA02);  // u of the previous chunk has read E
             if (!ok) break;
           }
-          put_tile(smem + C::OFF_AB, apk);
+          put_tile(apk);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(a_full);
@@ -887,11 +901,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(sd_free_da);
-          if (g > 0) {
-            ok = wwait(eb_empty, (g - 1) & 1, 0xA04);
-            if (!ok) break;
-          }
-          put_tile(smem + C::OFF_EB, epk);
+          ok = wwait(ab_free_a, g & 1, 0xA04);  // dV and qbar have read A
+          if (!ok) break;
+          put_tile(epk);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(e_full);
@@ -1040,7 +1052,7 @@ struct QCfg {
   static constexpr int NBAR = 2 * NSLOT + 20;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int SMEM = OFF_MISC + 16;
-  static constexpr int S_COL = 0, DA_COL = T, DS_COL = 2 * T, DQ_COL = 2 * T + T / 2;
+  static constexpr int S_COL = 0, DA_COL = T, DS_COL = 2 * T, DQ_COL = 3 * T;  // dS: two buffers of T/2
   static constexpr int TMEM_COLS = tmem_cols_for(DQ_COL + D);
   static_assert(PS == 128 && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
 };
@@ -1065,8 +1077,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto ring_empty = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
   const uint32_t b1 = bar0 + 8u * (2 * C::NSLOT);
   const uint32_t q_full = b1, q_empty = b1 + 8, g_full = b1 + 16, g_empty = b1 + 24, s_full = b1 + 32,
-                 s_free = b1 + 40, da_full = b1 + 48, da_free = b1 + 56, ds_full = b1 + 64, ds_empty = b1 + 72,
-                 dq_empty = b1 + 80, col_full0 = b1 + 88, col_empty0 = b1 + 104, drain = b1 + 120;
+                 s_free = b1 + 40, da_full = b1 + 48, da_free = b1 + 56, ds_full = b1 + 64, ds_empty0 = b1 + 72,
+                 dq_empty = b1 + 88, col_full0 = b1 + 96, col_empty0 = b1 + 112, drain = b1 + 128;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
   float* cols = reinterpret_cast<float*>(smem + C::OFF_COL);
@@ -1090,7 +1102,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(da_full, 1);
     mbar_init(da_free, kSoftWarps);
     mbar_init(ds_full, kSoftWarps);
-    mbar_init(ds_empty, 1);
+    mbar_init(ds_empty0, 1);
+    mbar_init(ds_empty0 + 8, 1);
     mbar_init(dq_empty, kSoftWarps);
     mbar_init(col_full0, 2);
     mbar_init(col_full0 + 8, 2);
@@ -1211,12 +1224,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         {
           const uint32_t kaddr = sRing + sK * C::KV_TILE;
+          const uint32_t dsb = C::DS_COL + (li & 1) * (T / 2);
 #pragma unroll
           for (int k = 0; k < T / 16; ++k)
-            umma_ts(tmem + C::DQ_COL, tmem + C::DS_COL + 8 * k, sdesc(kaddr + k * 2048, T * 128, 1024), idQ,
+            umma_ts(tmem + C::DQ_COL, tmem + dsb + 8 * k, sdesc(kaddr + k * 2048, T * 128, 1024), idQ,
                     (first_of_hp && k == 0) ? 0u : 1u);
         }
-        umma_commit(ds_empty);
+        umma_commit(ds_empty0 + 8 * (li & 1));
         umma_commit(ring_empty(sK));
         const bool last_of_hp = !more || newhead;
         if (last_of_hp) ++hp;
@@ -1285,7 +1299,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         ok = wwait(col_full0 + 8 * buf, (li >> 1) & 1, 0xF01);
         if (ok) ok = wwait(s_full, li & 1, 0xF02);
         if (ok) ok = wwait(da_full, li & 1, 0xF03);
-        if (ok && li > 0) ok = wwait(ds_empty, (li - 1) & 1, 0xF04);
+        // this tile's dS buffer was last read by dQ(i-2)
+        if (ok && li > 1) ok = wwait(ds_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xF04);
         if (!ok) break;
         tc_fence_after();
         const float* cl = cols + buf * 2 * T;
@@ -1312,7 +1327,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float a1 = ex2(fmaf(sv[2 * j + 1], c2, -cl[t + 1]));
             pk[j] = pack_bf16(a0 * (dv[2 * j] - cl[T + t]), a1 * (dv[2 * j + 1] - cl[T + t + 1]));
           }
-          tmem_st16(tmem + lane_off + C::DS_COL + col / 2, pk);
+          tmem_st16(tmem + lane_off + C::DS_COL + buf * (T / 2) + col / 2, pk);
         }
         tmem_st_wait();
         tc_fence_before();
@@ -1327,7 +1342,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int nn, hn;
         cur.peek_next(t0n, nn, hn);
         if (!more || hn != cur.h) {
-          ok = wwait(ds_empty, li & 1, 0xF05);
+          ok = wwait(ds_empty0 + 8 * buf, (li >> 1) & 1, 0xF05);
           if (!ok) break;
           tc_fence_after();
           float* dst = a.dq_partial + ((int64_t(wk) * a.H + cur.h) * a.P + p0) * D;
