@@ -609,28 +609,33 @@ template <int D, int P>
 struct TokCfg {
   static constexpr int NC = 128;
   static constexpr int NCH = P / NC;
-  static constexpr int KV_TILE = T * D * 2;
-  static constexpr int QG_CHUNK = NC * D * 2;
-  static constexpr int NQG = 4;  // ring of Q / G chunks: even slots Q, odd slots G
-  static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = KV_TILE;
-  static constexpr int OFF_QG = 2 * KV_TILE;
-  static constexpr int OFF_AB = OFF_QG + NQG * QG_CHUNK;  // A, then E = A o dA, of one chunk
+  static constexpr int SLOT = T * D * 2;  // one K, V, Q-chunk or G-chunk tile (NC == T)
+  static constexpr int NSLOT = 6;         // three pairs: (K, V) of a tile or (Q, G) of a chunk
+  static constexpr int OFF_SLOTS = 0;
+  static constexpr int OFF_AB = NSLOT * SLOT;  // A, then E = A o dA, of one chunk; epilogue staging
   static constexpr int OFF_STATS = OFF_AB + T * NC * 2;
   static constexpr int OFF_BAR = OFF_STATS + 2 * T * 4;
-  static constexpr int NBAR = 2 * NQG + 20;
+  static constexpr int NBAR = 2 * NSLOT + 20;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int SMEM = OFF_MISC + 16;
   static constexpr int SD_COL = 0, DV_COL = NC, U_COL = NC + D, QB_COL = NC + 2 * D;
   static constexpr int TMEM_COLS = tmem_cols_for(NC + 3 * D);
   static constexpr int HALF = NC / 2;
-  static_assert(TMEM_COLS <= 512 && SMEM <= 232448, "budget");
+  static_assert(NC == T && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
 };
+
+// Slot pairs rotate roles so the next tile's K and V load two chunks before
+// the tile ends: tile li keeps K, V in pair (li & 1); its chunks alternate
+// between pair 1 - (li & 1) and pair 2; pair 1 - (li & 1) is free after the
+// next-to-last chunk and takes tile li+1's K and V.
+__device__ __forceinline__ int tok_kv_pair(int li) { return li & 1; }
+__device__ __forceinline__ int tok_qg_pair(int li, int c) { return (c & 1) ? 2 : 1 - (li & 1); }
 
 template <int D, int P>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_bwd_tok_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                      const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmG, Args a,
+                      const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmG,
+                      const __grid_constant__ CUtensorMap tmDK, const __grid_constant__ CUtensorMap tmDV, Args a,
                       const float* __restrict__ lse, float* __restrict__ Dco, __nv_bfloat16* __restrict__ dK,
                       __nv_bfloat16* __restrict__ dV) {
   using C = TokCfg<D, P>;
@@ -642,15 +647,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t sK = sbase + C::OFF_K, sV = sbase + C::OFF_V, sQG = sbase + C::OFF_QG, sAB = sbase + C::OFF_AB;
+  const uint32_t sSlots = sbase + C::OFF_SLOTS, sAB = sbase + C::OFF_AB;
+  auto slot_addr = [&](int s) { return sSlots + uint32_t(s) * C::SLOT; };
   const uint32_t bar0 = sbase + C::OFF_BAR;
-  auto qg_full = [&](int s) { return bar0 + 8u * s; };
-  auto qg_empty = [&](int s) { return bar0 + 8u * (C::NQG + s); };
-  const uint32_t b1 = bar0 + 8u * (2 * C::NQG);
-  const uint32_t k_full = b1, k_empty = b1 + 8, v_full = b1 + 16, v_empty = b1 + 24, s_full = b1 + 32,
-                 sd_free_s = b1 + 40, da_full = b1 + 48, sd_free_da = b1 + 56, a_full = b1 + 64,
-                 ab_free_a = b1 + 72, e_full = b1 + 80, ab_free_e = b1 + 88, acc_full = b1 + 96,
-                 acc_empty = b1 + 104, st_ready = b1 + 112, st_used = b1 + 120, drain = b1 + 128;
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
+  const uint32_t b1 = bar0 + 8u * (2 * C::NSLOT);
+  const uint32_t s_full = b1, sd_free_s = b1 + 8, da_full = b1 + 16, sd_free_da = b1 + 24, a_full = b1 + 32,
+                 ab_free_a = b1 + 40, e_full = b1 + 48, ab_free_e = b1 + 56, acc_full = b1 + 64,
+                 acc_empty = b1 + 72, st_ready = b1 + 80, st_used = b1 + 88, epi_ready = b1 + 96, epi_free = b1 + 104,
+                 drain = b1 + 112;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
   const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
@@ -659,14 +665,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
   const int ntiles = int(te - tb);
   if (threadIdx.x == 0) {
-    for (int s = 0; s < C::NQG; ++s) {
-      mbar_init(qg_full(s), 1);
-      mbar_init(qg_empty(s), 1);
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
     }
-    mbar_init(k_full, 1);
-    mbar_init(k_empty, 1);
-    mbar_init(v_full, 1);
-    mbar_init(v_empty, 1);
     mbar_init(s_full, 1);
     mbar_init(sd_free_s, kSoftWarps);
     mbar_init(da_full, 1);
@@ -679,6 +681,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(acc_empty, kSoftWarps);
     mbar_init(st_ready, kSoftWarps);
     mbar_init(st_used, kSoftWarps);
+    mbar_init(epi_ready, kSoftWarps);
+    mbar_init(epi_free, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -696,91 +700,87 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmV);
       tma_prefetch_desc(&tmQ);
       tma_prefetch_desc(&tmG);
-      TileWalker it(a, tb, te, T);
-      uint32_t e = 0;
+      TileWalker it(a, tb, te, T), nx(a, tb, te, T);
+      nx.next();
+      int uses[C::NSLOT] = {0, 0, 0, 0, 0, 0};
       bool ok = true;
+      // box origin (64*dh, c1, c2): K / V maps are (d, head, token); Q / G maps
+      // are (d, prototype, head) and (d, prototype, user*H + head)
+      auto load = [&](int s, const CUtensorMap* map, int c1, int c2) {
+        if (uses[s] > 0) ok = ok && mbar_wait(empty_bar(s), (uses[s] - 1) & 1, abort_flag, a.ws, 0x801);
+        if (!ok) return;
+        ++uses[s];
+        mbar_arrive_expect_tx(full_bar(s), C::SLOT);
+#pragma unroll
+        for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(slot_addr(s) + dh * T * 128, map, full_bar(s), 64 * dh, c1, c2);
+      };
+      auto load_kv = [&](int li, const TileWalker& w) {
+        const int pr = tok_kv_pair(li);
+        load(2 * pr, &tmK, w.h, int(w.tok0));
+        load(2 * pr + 1, &tmV, w.h, int(w.tok0));
+      };
+      load_kv(0, it);
       for (int li = 0; li < ntiles && ok; ++li) {
-        if (li > 0) ok = mbar_wait(k_empty, (li - 1) & 1, abort_flag, a.ws, 0x801);
-        if (!ok) break;
-        mbar_arrive_expect_tx(k_full, C::KV_TILE);
-#pragma unroll
-        for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sK + dh * T * 128, &tmK, k_full, 64 * dh, it.h, int(it.tok0));
         for (int c = 0; c < C::NCH && ok; ++c) {
-#pragma unroll
-          for (int g = 0; g < 2; ++g) {
-            const int s = int(e % C::NQG);
-            if (e >= uint32_t(C::NQG)) ok = mbar_wait(qg_empty(s), ((e / C::NQG) + 1) & 1, abort_flag, a.ws, 0x802);
-            if (!ok) break;
-            mbar_arrive_expect_tx(qg_full(s), C::QG_CHUNK);
-            const int ghead = g ? int(it.b) * a.H + it.h : it.h;  // G copy is [B*H][P][D]
-#pragma unroll
-            for (int dh = 0; dh < D / 64; ++dh)
-              tma_load_3d(sQG + s * C::QG_CHUNK + dh * C::NC * 128, g ? &tmG : &tmQ, qg_full(s), 64 * dh, c * C::NC,
-                          ghead);
-            ++e;
-          }
-          if (c == 0 && ok) {  // V right after the first chunk: dA of chunk 0 needs it next
-            if (li > 0) ok = mbar_wait(v_empty, (li - 1) & 1, abort_flag, a.ws, 0x803);
-            if (!ok) break;
-            mbar_arrive_expect_tx(v_full, C::KV_TILE);
-#pragma unroll
-            for (int dh = 0; dh < D / 64; ++dh)
-              tma_load_3d(sV + dh * T * 128, &tmV, v_full, 64 * dh, it.h, int(it.tok0));
-          }
+          const int pr = tok_qg_pair(li, c);
+          load(2 * pr, &tmQ, c * C::NC, it.h);
+          load(2 * pr + 1, &tmG, c * C::NC, int(it.b) * a.H + it.h);
+          if (c == C::NCH - 1 && li + 1 < ntiles) load_kv(li + 1, nx);
         }
         it.next();
+        nx.next();
       }
       if (!ok) {
-        for (uint32_t k = (e > uint32_t(C::NQG) ? e - C::NQG : 0); k < e; ++k)
-          mbar_wait_bounded(qg_full(int(k % C::NQG)), (k / C::NQG) & 1, 200000000ull);
-        mbar_wait_bounded(k_full, (ntiles - 1) & 1, 200000000ull);
-        mbar_wait_bounded(v_full, (ntiles - 1) & 1, 200000000ull);
+        for (int s = 0; s < C::NSLOT; ++s)
+          if (uses[s] > 0) mbar_wait_bounded(full_bar(s), (uses[s] - 1) & 1, 200000000ull);
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- UMMA issuer
-      // Order per chunk g: dA_g, dV_g + qbar_g, S_{g+1}, u_g.  S of the next chunk
-      // runs while the softmax warps wait to put E_g where A_g was.
+      // Per chunk g: dA_g, dV_g + qbar_g, S_{g+1}, u_g.
       constexpr uint32_t idS = idesc_bf16(128, C::NC, 0, 0);  // [tok x chunk], K = d
       constexpr uint32_t idTD = idesc_bf16(128, D, 0, 1);     // [tok x d], K = chunk prototypes
       bool ok = true;
+      int uses[C::NSLOT] = {0, 0, 0, 0, 0, 0};
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
       };
+      auto wfull = [&](int s, uint32_t site) {
+        wt(full_bar(s), uses[s] & 1, site);
+        ++uses[s];
+      };
       const uint32_t nchunks = uint32_t(ntiles) * C::NCH;
       auto issue_S = [&](uint32_t g) {
-        const uint32_t sq = (2 * g) % C::NQG;
-        const uint32_t aQ = sQG + sq * C::QG_CHUNK;
+        const int li = int(g / C::NCH), c = int(g % C::NCH);
+        const uint32_t aK = slot_addr(2 * tok_kv_pair(li)), aQ = slot_addr(2 * tok_qg_pair(li, c));
 #pragma unroll
         for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + C::SD_COL, sdesc(sK + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+          umma_ss(tmem + C::SD_COL, sdesc(aK + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
                   sdesc(aQ + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
         umma_commit(s_full);
-        if (g % C::NCH == C::NCH - 1) umma_commit(k_empty);  // last S of the tile
+        if (c == C::NCH - 1) umma_commit(empty_bar(2 * tok_kv_pair(li)));  // last S: K free
       };
-      // S_0
-      wt(k_full, 0, 0x901);
-      wt(qg_full(0), 0, 0x902);
+      wfull(2 * tok_kv_pair(0), 0x901);
+      wfull(2 * tok_qg_pair(0, 0), 0x902);
       if (ok) {
         tc_fence_after();
         issue_S(0);
       }
       for (uint32_t g = 0; g < nchunks && ok; ++g) {
-        const uint32_t li = g / C::NCH, c = g % C::NCH;
-        const uint32_t eQ = 2 * g, eG = eQ + 1;
-        const int sq = int(eQ % C::NQG), sg = int(eG % C::NQG);
-        const uint32_t aQ = sQG + sq * C::QG_CHUNK, aG = sQG + sg * C::QG_CHUNK;
-        // ---- dA_g = V G_g^T (into the S/dA columns once S_g was read)
-        if (c == 0) wt(v_full, li & 1, 0x903);
-        wt(qg_full(sg), (eG / C::NQG) & 1, 0x904);
+        const int li = int(g / C::NCH), c = int(g % C::NCH);
+        const int kvp = tok_kv_pair(li), qgp = tok_qg_pair(li, c);
+        const uint32_t aV = slot_addr(2 * kvp + 1), aQ = slot_addr(2 * qgp), aG = slot_addr(2 * qgp + 1);
+        // ---- dA_g = V G_g^T
+        if (c == 0) wfull(2 * kvp + 1, 0x903);
+        wfull(2 * qgp + 1, 0x904);
         wt(sd_free_s, g & 1, 0x905);
         if (!ok) break;
         tc_fence_after();
 #pragma unroll
         for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + C::SD_COL, sdesc(sV + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
+          umma_ss(tmem + C::SD_COL, sdesc(aV + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
                   sdesc(aG + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
         umma_commit(da_full);
-        if (c == C::NCH - 1) umma_commit(v_empty);
+        if (c == C::NCH - 1) umma_commit(empty_bar(2 * kvp + 1));  // last dA: V free
         // ---- dV += A G_g, qbar += A Q_g
         wt(a_full, g & 1, 0x906);
         if (c == 0 && li > 0) wt(acc_empty, (li - 1) & 1, 0x907);
@@ -794,12 +794,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_ss(tmem + C::QB_COL, ad, sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, acc);
         }
         umma_commit(ab_free_a);
-        umma_commit(qg_empty(sg));
+        umma_commit(empty_bar(2 * qgp + 1));  // G chunk free
         // ---- S_{g+1}
         if (g + 1 < nchunks) {
           const uint32_t gn = g + 1;
-          if (gn % C::NCH == 0) wt(k_full, (gn / C::NCH) & 1, 0x908);
-          wt(qg_full(int((2 * gn) % C::NQG)), ((2 * gn) / C::NQG) & 1, 0x909);
+          const int lin = int(gn / C::NCH), cn = int(gn % C::NCH);
+          if (cn == 0) wfull(2 * tok_kv_pair(lin), 0x908);
+          wfull(2 * tok_qg_pair(lin, cn), 0x909);
           wt(sd_free_da, g & 1, 0x90A);
           if (!ok) break;
           tc_fence_after();
@@ -814,7 +815,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_ss(tmem + C::U_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
                   sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, (c == 0 && k == 0) ? 0u : 1u);
         umma_commit(ab_free_e);
-        umma_commit(qg_empty(sq));
+        umma_commit(empty_bar(2 * qgp));  // Q chunk free
         if (c == C::NCH - 1) umma_commit(acc_full);
       }
       umma_commit(drain);
@@ -831,6 +832,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
       };
       uint32_t g = 0;
+      int epi = 0;  // staged epilogue stores so far
       auto put_tile = [&](const uint32_t* pk) {
         uint8_t* rowp = smem + C::OFF_AB + row * 128;
 #pragma unroll
@@ -840,6 +842,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           *reinterpret_cast<uint4*>(rowp + blk * (T * 128) + ((chunk ^ (row & 7)) << 4)) =
               make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
         }
+      };
+      // one staged [128 tokens][D] bf16 tile in AB -> global through TMA
+      auto stage_and_store = [&](const CUtensorMap* map, const TileWalker& w) -> bool {
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(epi_ready);
+        if (warp == kSoftWarp0 && lane == 0) {
+          if (mbar_wait(epi_ready, epi & 1, abort_flag, a.ws, 0xA08)) {
+#pragma unroll
+            for (int dh = 0; dh < D / 64; ++dh) tma_store_3d(map, sAB + dh * T * 128, 64 * dh, w.h, int(w.tok0));
+            bulk_commit_group();
+            bulk_wait_read_all();
+          }
+          mbar_arrive(epi_free);
+        }
+        const bool r = wwait(epi_free, epi & 1, 0xA09);
+        ++epi;
+        return r;
       };
       float lse_cur = row < cur.n ? lse[(cur.tok0 + row) * a.H + cur.h] : 0.f;
       for (int li = 0; li < ntiles && ok; ++li) {
@@ -923,11 +943,45 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(st_used);
         if (sw == 0 && valid) Dco[tok * a.H + cur.h] = Dv;
-        // epilogue: dV and dK = scale (u - D qbar) for this warpgroup's column half
+        // epilogue: dV and dK = scale (u - D qbar); this warpgroup owns columns [sw*D/2, +D/2)
         ok = wwait(acc_full, li & 1, 0xA07);
         if (!ok) break;
         tc_fence_after();
-        {
+        const bool whole = cur.n == T;  // a full tile is stored by TMA; a ragged tail row by row
+        uint8_t* rowp = smem + C::OFF_AB + row * 128;
+        auto put_half = [&](const float* x, int cc) {  // 32 columns [sw*D/2 + cc, +32) of this row
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int col = sw * (D / 2) + cc + 8 * k;
+            const int dh = col >> 6, chunk = (col & 63) >> 3;
+            *reinterpret_cast<uint4*>(rowp + dh * (T * 128) + ((chunk ^ (row & 7)) << 4)) =
+                make_uint4(pack_bf16(x[8 * k], x[8 * k + 1]), pack_bf16(x[8 * k + 2], x[8 * k + 3]),
+                           pack_bf16(x[8 * k + 4], x[8 * k + 5]), pack_bf16(x[8 * k + 6], x[8 * k + 7]));
+          }
+        };
+        if (whole) {
+          float x[32];
+#pragma unroll
+          for (int cc = 0; cc < D / 2; cc += 32) {
+            tmem_ld32(tmem + lane_off + C::DV_COL + sw * (D / 2) + cc, x);
+            tmem_ld_wait();
+            put_half(x, cc);
+          }
+          ok = stage_and_store(&tmDV, cur);
+          if (!ok) break;
+          float uu[32], qb[32];
+#pragma unroll
+          for (int cc = 0; cc < D / 2; cc += 32) {
+            tmem_ld32(tmem + lane_off + C::U_COL + sw * (D / 2) + cc, uu);
+            tmem_ld32(tmem + lane_off + C::QB_COL + sw * (D / 2) + cc, qb);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) uu[j] = a.scale * fmaf(-Dv, qb[j], uu[j]);
+            put_half(uu, cc);
+          }
+          ok = stage_and_store(&tmDK, cur);
+          if (!ok) break;
+        } else {
           __nv_bfloat16* dvr = dV + (tok * a.H + cur.h) * int64_t(D) + sw * (D / 2);
           store_row_bf16<D / 2>(tmem + lane_off + C::DV_COL + sw * (D / 2), dvr, 1.f, valid);
           __nv_bfloat16* dkr = dK + (tok * a.H + cur.h) * int64_t(D) + sw * (D / 2);
@@ -955,6 +1009,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(acc_empty);
         cur.next();
       }
+      if (warp == kSoftWarp0 && lane == 0) bulk_wait_all();  // stores complete before exit
     }
   }
   __syncthreads();
@@ -963,12 +1018,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
 }
-
-}  // namespace tcb
-}  // namespace sa
-
-namespace sa {
-namespace tcb {
 
 // dsketch fp32 -> bf16 copy in the workspace, the layout TMA streams ([B*H][P][D])
 __global__ void to_bf16_kernel(const float* __restrict__ src, __nv_bfloat16* __restrict__ dst, int64_t n8,
@@ -986,14 +1035,15 @@ template <int D, int P>
 static cudaError_t launch_tok_t(const Args& a, int W, const __nv_bfloat16* gbf, const float* lse, float* Dco,
                                 void* dK, void* dV, cudaStream_t st) {
   using C = TokCfg<D, P>;
-  CUtensorMap tk, tv, tq, tg;
+  CUtensorMap tk, tv, tq, tg, tdk, tdv;
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
-      !make_q_map(&tq, a.Q, a.H, a.P, D, C::NC) || !make_q_map(&tg, gbf, a.B * a.H, a.P, D, C::NC))
+      !make_q_map(&tq, a.Q, a.H, a.P, D, C::NC) || !make_q_map(&tg, gbf, a.B * a.H, a.P, D, C::NC) ||
+      !make_kv_map(&tdk, dK, a.N, a.H, D) || !make_kv_map(&tdv, dV, a.N, a.H, D))
     return cudaErrorInvalidValue;
   auto fn = &tc_bwd_tok_kernel<D, P>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
-  fn<<<W, kThreads, C::SMEM, st>>>(tk, tv, tq, tg, a, lse, Dco, static_cast<__nv_bfloat16*>(dK),
+  fn<<<W, kThreads, C::SMEM, st>>>(tk, tv, tq, tg, tdk, tdv, a, lse, Dco, static_cast<__nv_bfloat16*>(dK),
                                    static_cast<__nv_bfloat16*>(dV));
   return cudaGetLastError();
 }
