@@ -1226,6 +1226,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_ss(tmem + dcol, sdesc(aop + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024),
                   sdesc(bop + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024), idPT, k > 0 ? 1u : 0u);
       };
+      // Issue order: S(0), dA(0); then per tile i: S(i+1), dA(i+1), dQ(i), so the
+      // next tile's scores are ready when the softmax warps finish tile i.
+      auto issue_dA = [&](int li, bool seg_first) -> bool {
+        const uint32_t eV = 2u * li + 1;
+        const int sV = int(eV % C::NSLOT);
+        if (seg_first) {
+          wt(g_full, gc & 1, 0xD03);
+          ++gc;
+        }
+        wt(ring_full(sV), (eV / C::NSLOT) & 1, 0xD04);
+        if (li > 0) wt(da_free, (li - 1) & 1, 0xD05);
+        if (!ok) return false;
+        tc_fence_after();
+        issue_pt(C::DA_COL, sG, sRing + sV * C::KV_TILE);
+        umma_commit(da_full);
+        umma_commit(ring_empty(sV));
+        return true;
+      };
       wt(q_full, 0, 0xD01);
       wt(ring_full(0), 0, 0xD02);
       if (ok) {
@@ -1233,28 +1251,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         issue_pt(C::S_COL, sQ, sRing);
         umma_commit(s_full);
         if (ntiles == 1 || nxt.h != cur.h) umma_commit(q_empty);
+        issue_dA(0, cur.seg_first);
+        if (cur.seg_last) umma_commit(g_empty);
       }
       bool first_of_hp = true;
       for (int li = 0; li < ntiles && ok; ++li) {
-        const uint32_t eK = 2u * li, eV = eK + 1;
-        const int sK = int(eK % C::NSLOT), sV = int(eV % C::NSLOT);
-        // ---- dA(i) = G_r V(i)^T
-        if (cur.seg_first) {
-          wt(g_full, gc & 1, 0xD03);
-          ++gc;
-        }
-        wt(ring_full(sV), (eV / C::NSLOT) & 1, 0xD04);
-        if (li > 0) wt(da_free, (li - 1) & 1, 0xD05);
-        if (!ok) break;
-        tc_fence_after();
-        issue_pt(C::DA_COL, sG, sRing + sV * C::KV_TILE);
-        umma_commit(da_full);
-        umma_commit(ring_empty(sV));
-        if (cur.seg_last) umma_commit(g_empty);
-        // ---- S(i+1) while the softmax warps work on tile i
+        const uint32_t eK = 2u * li;
+        const int sK = int(eK % C::NSLOT);
         const bool more = li + 1 < ntiles;
         const bool newhead = more && nxt.h != cur.h;
         if (more) {
+          // ---- S(i+1) = Q_r K(i+1)^T once the softmax warps hold S(i)
           if (newhead) {
             ++hc;
             wt(q_full, hc & 1, 0xD06);
@@ -1266,8 +1273,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_pt(C::S_COL, sQ, sRing + ((eK + 2) % C::NSLOT) * C::KV_TILE);
           umma_commit(s_full);
           if (li + 2 >= ntiles || nx2.h != nxt.h) umma_commit(q_empty);
+          // ---- dA(i+1) = G_r V(i+1)^T once they hold dA(i)
+          if (!issue_dA(li + 1, nxt.seg_first)) break;
+          if (nxt.seg_last) umma_commit(g_empty);
         }
-        // ---- dQ += dS K(i), dS read from TMEM
+        // ---- dQ += dS(i) K(i), dS read from TMEM
         wt(ds_full, li & 1, 0xD09);
         if (first_of_hp && hp > 0) wt(dq_empty, (hp - 1) & 1, 0xD0A);
         if (!ok) break;
