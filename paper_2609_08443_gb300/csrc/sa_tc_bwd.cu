@@ -1093,7 +1093,7 @@ template <int D, int PS>
 struct QCfg {
   static constexpr int KV_TILE = T * D * 2;
   static constexpr int QB = PS * D * 2;
-  static constexpr int NSLOT = 4;
+  static constexpr int NSLOT = 5;  // K and V tiles alternate over 5 slots: 2.5 tiles of lookahead
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_G = QB;
   static constexpr int OFF_RING = 2 * QB;
@@ -1364,28 +1364,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         tc_fence_after();
         const float* cl = cols + buf * 2 * T;
+        float sv[64], dv[64];  // this warpgroup's 64 token columns of S and dA
+        tmem_ld32(tmem + lane_off + C::S_COL + 64 * sw, sv);
+        tmem_ld32(tmem + lane_off + C::S_COL + 64 * sw + 32, sv + 32);
+        tmem_ld32(tmem + lane_off + C::DA_COL + 64 * sw, dv);
+        tmem_ld32(tmem + lane_off + C::DA_COL + 64 * sw + 32, dv + 32);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {  // the next tile's S and dA may now be written
+          mbar_arrive(s_free);
+          mbar_arrive(da_free);
+        }
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           const int col = 64 * sw + 32 * c;
-          float sv[32], dv[32];
-          tmem_ld32(tmem + lane_off + C::S_COL + col, sv);
-          tmem_ld32(tmem + lane_off + C::DA_COL + col, dv);
-          tmem_ld_wait();
-          if (c == 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) {
-              mbar_arrive(s_free);
-              mbar_arrive(da_free);
-            }
-          }
           uint32_t pk[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const int t = col + 2 * j;
-            const float a0 = ex2(fmaf(sv[2 * j], c2, -cl[t]));
-            const float a1 = ex2(fmaf(sv[2 * j + 1], c2, -cl[t + 1]));
-            pk[j] = pack_bf16(a0 * (dv[2 * j] - cl[T + t]), a1 * (dv[2 * j + 1] - cl[T + t + 1]));
+            const int jj = 32 * c + 2 * j;
+            const float a0 = ex2(fmaf(sv[jj], c2, -cl[t]));
+            const float a1 = ex2(fmaf(sv[jj + 1], c2, -cl[t + 1]));
+            pk[j] = pack_bf16(a0 * (dv[jj] - cl[T + t]), a1 * (dv[jj + 1] - cl[T + t + 1]));
           }
           tmem_st16(tmem + lane_off + C::DS_COL + buf * (T / 2) + col / 2, pk);
         }

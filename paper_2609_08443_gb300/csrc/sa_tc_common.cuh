@@ -28,6 +28,7 @@ struct TileWalker {
   int64_t tph, t, tb, te;
   int h, b;
   int64_t k, nk, tok0, seg0, seg1;
+  int64_t cub, Lb;  // cu[b] and L_b of the current user, read once per segment
   int n;
   bool seg_first, seg_last;
 
@@ -44,12 +45,13 @@ struct TileWalker {
     seg1 = r.seg1;
     nk = seg1 - seg0;
     k = t - seg0;
+    cub = int64_t(cu[b]);
+    Lb = int64_t(cu[b + 1]) - cub;
     fields();
   }
   __device__ void fields() {
-    const int64_t L = int64_t(cu[b + 1]) - int64_t(cu[b]);
-    tok0 = int64_t(cu[b]) + k * Tt;
-    const int64_t left = L - k * Tt;
+    tok0 = cub + k * Tt;
+    const int64_t left = Lb - k * Tt;
     n = int(left < Tt ? left : Tt);
     seg_first = (k == 0) || (t == tb);
     seg_last = (k == nk - 1) || (t == te - 1);
@@ -63,9 +65,8 @@ struct TileWalker {
       return;
     }
     if (k + 1 < nk) {
-      const int64_t L = int64_t(cu[b + 1]) - int64_t(cu[b]);
       tok0_n = tok0 + Tt;
-      const int64_t left = L - (k + 1) * Tt;
+      const int64_t left = Lb - (k + 1) * Tt;
       n_n = int(left < Tt ? left : Tt);
       h_n = h;
     } else {
