@@ -114,15 +114,18 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// D[tmem] (+)= A[smem] * B[smem], kind::f16 (bf16 inputs, fp32 accumulate)
+// D[tmem] (+)= A[smem] * B[smem], kind::f16 (bf16 inputs, fp32 accumulate).
+// No "memory" clobber: the issuing thread touches no memory the MMA reads, and
+// volatile asm keeps its order against the mbarrier waits and tcgen05 fences,
+// so the compiler can keep addresses and descriptors in registers between
+// issues (an issue must cost far less than the 64 cycles of a 128x128x16 MMA).
 __device__ __forceinline__ void umma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                         uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
 }
 // D[tmem] (+)= A[tmem] * B[smem]: A is M x K with M on TMEM lanes and two bf16
 // values per 32-bit column (lower K index in the low half).
@@ -132,8 +135,7 @@ __device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate));
 }
 // mbarrier arrives once every tcgen05 op issued so far by this thread is done
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
@@ -182,6 +184,12 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo_bytes, ui
   d |= uint64_t(1) << 46;  // descriptor version for tcgen05
   d |= uint64_t(2) << 61;  // 128-byte swizzle
   return d;
+}
+
+// The same descriptor with its start address moved by `bytes` (a multiple of
+// 16; the 14-bit address field cannot overflow inside 228 KB of shared memory).
+__host__ __device__ __forceinline__ uint64_t sdesc_add(uint64_t desc, uint32_t bytes) {
+  return desc + uint64_t(bytes >> 4);
 }
 
 // Instruction descriptor, kind::f16: bf16 A and B, fp32 D; a_mn / b_mn select

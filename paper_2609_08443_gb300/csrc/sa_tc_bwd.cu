@@ -1376,17 +1376,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive(s_free);
           mbar_arrive(da_free);
         }
+        // per-token values as 16-byte broadcasts: one shared-memory wavefront per 4 tokens
+        const float4* cl4 = reinterpret_cast<const float4*>(cl);
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           const int col = 64 * sw + 32 * c;
           uint32_t pk[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int t = col + 2 * j;
-            const int jj = 32 * c + 2 * j;
-            const float a0 = ex2(fmaf(sv[jj], c2, -cl[t]));
-            const float a1 = ex2(fmaf(sv[jj + 1], c2, -cl[t + 1]));
-            pk[j] = pack_bf16(a0 * (dv[jj] - cl[T + t]), a1 * (dv[jj + 1] - cl[T + t + 1]));
+          for (int j4 = 0; j4 < 8; ++j4) {
+            const float4 l4 = cl4[(col >> 2) + j4];
+            const float4 d4 = cl4[((T + col) >> 2) + j4];
+            const int jj = 32 * c + 4 * j4;
+            const float a0 = ex2(fmaf(sv[jj], c2, -l4.x)), a1 = ex2(fmaf(sv[jj + 1], c2, -l4.y));
+            const float a2 = ex2(fmaf(sv[jj + 2], c2, -l4.z)), a3 = ex2(fmaf(sv[jj + 3], c2, -l4.w));
+            pk[2 * j4] = pack_bf16(a0 * (dv[jj] - d4.x), a1 * (dv[jj + 1] - d4.y));
+            pk[2 * j4 + 1] = pack_bf16(a2 * (dv[jj + 2] - d4.z), a3 * (dv[jj + 3] - d4.w));
           }
           tmem_st16(tmem + lane_off + C::DS_COL + buf * (T / 2) + col / 2, pk);
         }
