@@ -610,7 +610,7 @@ struct TokCfg {
   static constexpr int NC = 128;
   static constexpr int NCH = P / NC;
   static constexpr int SLOT = T * D * 2;  // one K, V, Q-chunk or G-chunk tile (NC == T)
-  static constexpr int NSLOT = 6;         // three pairs: (K, V) of a tile or (Q, G) of a chunk
+  static constexpr int NSLOT = 6;         // three pairs: (K, V) of a tile or (G, Q) of a chunk
   static constexpr int OFF_SLOTS = 0;
   static constexpr int OFF_AB = NSLOT * SLOT;  // A, then E = A o dA, of one chunk; epilogue staging
   static constexpr int OFF_STATS = OFF_AB + T * NC * 2;
@@ -618,7 +618,8 @@ struct TokCfg {
   static constexpr int NBAR = 2 * NSLOT + 20;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int SMEM = OFF_MISC + 16;
-  static constexpr int SD_COL = 0, DV_COL = NC, U_COL = NC + D, QB_COL = NC + 2 * D;
+  // dV and qbar side by side: one N = 2D MMA against the adjacent G, Q chunks
+  static constexpr int SD_COL = 0, DV_COL = NC, QB_COL = NC + D, U_COL = NC + 2 * D;
   static constexpr int TMEM_COLS = tmem_cols_for(NC + 3 * D);
   static constexpr int HALF = NC / 2;
   static_assert(NC == T && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
@@ -627,7 +628,9 @@ struct TokCfg {
 // Slot pairs rotate roles so the next tile's K and V load two chunks before
 // the tile ends: tile li keeps K, V in pair (li & 1); its chunks alternate
 // between pair 1 - (li & 1) and pair 2; pair 1 - (li & 1) is free after the
-// next-to-last chunk and takes tile li+1's K and V.
+// next-to-last chunk and takes tile li+1's K and V.  A chunk pair holds G in
+// its first slot and Q in the second, so the four 64-column blocks of G and Q
+// sit at one stride and [G | Q] is a single N = 2D operand.
 __device__ __forceinline__ int tok_kv_pair(int li) { return li & 1; }
 __device__ __forceinline__ int tok_qg_pair(int li, int c) { return (c & 1) ? 2 : 1 - (li & 1); }
 
@@ -723,8 +726,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int li = 0; li < ntiles && ok; ++li) {
         for (int c = 0; c < C::NCH && ok; ++c) {
           const int pr = tok_qg_pair(li, c);
-          load(2 * pr, &tmQ, c * C::NC, it.h);
-          load(2 * pr + 1, &tmG, c * C::NC, int(it.b) * a.H + it.h);
+          load(2 * pr + 1, &tmQ, c * C::NC, it.h);
+          load(2 * pr, &tmG, c * C::NC, int(it.b) * a.H + it.h);
           if (c == C::NCH - 1 && li + 1 < ntiles) load_kv(li + 1, nx);
         }
         it.next();
@@ -736,9 +739,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- UMMA issuer
-      // Per chunk g: dA_g, dV_g + qbar_g, S_{g+1}, u_g.
-      constexpr uint32_t idS = idesc_bf16(128, C::NC, 0, 0);  // [tok x chunk], K = d
-      constexpr uint32_t idTD = idesc_bf16(128, D, 0, 1);     // [tok x d], K = chunk prototypes
+      // Per chunk g: dA_g, [dV | qbar]_g, S_{g+1}, u_g.  Shared-memory
+      // descriptors are built once per operand and stepped by constant offsets,
+      // so the issue loop carries no address arithmetic.
+      constexpr uint32_t idS = idesc_bf16(128, C::NC, 0, 0);    // [tok x chunk], K = d
+      constexpr uint32_t idGQ = idesc_bf16(128, 2 * D, 0, 1);   // [tok x (d | d)], K = chunk prototypes
+      constexpr uint32_t idU = idesc_bf16(128, D, 0, 1);        // [tok x d], K = chunk prototypes
       bool ok = true;
       int uses[C::NSLOT] = {0, 0, 0, 0, 0, 0};
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
@@ -748,19 +754,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         wt(full_bar(s), uses[s] & 1, site);
         ++uses[s];
       };
+      // K-major [128 rows x D] operand: K step k at +(k / 4) * 128 rows + (k % 4) * 32 B
+      auto kmaj = [](uint32_t addr) { return sdesc(addr, 16, 1024); };
+      auto kstep = [](int k) { return uint32_t((k >> 2) * (T * 128) + (k & 3) * 32); };
+      const uint64_t dAB = kmaj(sAB);
       const uint32_t nchunks = uint32_t(ntiles) * C::NCH;
       auto issue_S = [&](uint32_t g) {
         const int li = int(g / C::NCH), c = int(g % C::NCH);
-        const uint32_t aK = slot_addr(2 * tok_kv_pair(li)), aQ = slot_addr(2 * tok_qg_pair(li, c));
+        const uint64_t dK = kmaj(slot_addr(2 * tok_kv_pair(li))), dQ = kmaj(slot_addr(2 * tok_qg_pair(li, c) + 1));
 #pragma unroll
         for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + C::SD_COL, sdesc(aK + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                  sdesc(aQ + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
+          umma_ss(tmem + C::SD_COL, sdesc_add(dK, kstep(k)), sdesc_add(dQ, kstep(k)), idS, k > 0 ? 1u : 0u);
         umma_commit(s_full);
         if (c == C::NCH - 1) umma_commit(empty_bar(2 * tok_kv_pair(li)));  // last S: K free
       };
       wfull(2 * tok_kv_pair(0), 0x901);
-      wfull(2 * tok_qg_pair(0, 0), 0x902);
+      wfull(2 * tok_qg_pair(0, 0) + 1, 0x902);
       if (ok) {
         tc_fence_after();
         issue_S(0);
@@ -768,39 +777,41 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (uint32_t g = 0; g < nchunks && ok; ++g) {
         const int li = int(g / C::NCH), c = int(g % C::NCH);
         const int kvp = tok_kv_pair(li), qgp = tok_qg_pair(li, c);
-        const uint32_t aV = slot_addr(2 * kvp + 1), aQ = slot_addr(2 * qgp), aG = slot_addr(2 * qgp + 1);
+        const uint32_t aG = slot_addr(2 * qgp), aQ = slot_addr(2 * qgp + 1);
         // ---- dA_g = V G_g^T
         if (c == 0) wfull(2 * kvp + 1, 0x903);
-        wfull(2 * qgp + 1, 0x904);
+        wfull(2 * qgp, 0x904);
         wt(sd_free_s, g & 1, 0x905);
         if (!ok) break;
         tc_fence_after();
+        {
+          const uint64_t dV = kmaj(slot_addr(2 * kvp + 1)), dG = kmaj(aG);
 #pragma unroll
-        for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + C::SD_COL, sdesc(aV + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                  sdesc(aG + (k >> 2) * (C::NC * 128) + (k & 3) * 32, 16, 1024), idS, k > 0 ? 1u : 0u);
+          for (int k = 0; k < D / 16; ++k)
+            umma_ss(tmem + C::SD_COL, sdesc_add(dV, kstep(k)), sdesc_add(dG, kstep(k)), idS, k > 0 ? 1u : 0u);
+        }
         umma_commit(da_full);
         if (c == C::NCH - 1) umma_commit(empty_bar(2 * kvp + 1));  // last dA: V free
-        // ---- dV += A G_g, qbar += A Q_g
+        // ---- [dV | qbar] += A [G_g | Q_g]
         wt(a_full, g & 1, 0x906);
         if (c == 0 && li > 0) wt(acc_empty, (li - 1) & 1, 0x907);
         if (!ok) break;
         tc_fence_after();
+        {
+          const uint64_t dGQ = sdesc(aG, C::NC * 128, 1024);  // MN-major, 64-column blocks 16 KB apart
 #pragma unroll
-        for (int k = 0; k < C::NC / 16; ++k) {
-          const uint64_t ad = sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024);
-          const uint32_t acc = (c == 0 && k == 0) ? 0u : 1u;
-          umma_ss(tmem + C::DV_COL, ad, sdesc(aG + k * 2048, C::NC * 128, 1024), idTD, acc);
-          umma_ss(tmem + C::QB_COL, ad, sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, acc);
+          for (int k = 0; k < C::NC / 16; ++k)
+            umma_ss(tmem + C::DV_COL, sdesc_add(dAB, kstep(k)), sdesc_add(dGQ, k * 2048), idGQ,
+                    (c == 0 && k == 0) ? 0u : 1u);
         }
         umma_commit(ab_free_a);
-        umma_commit(empty_bar(2 * qgp + 1));  // G chunk free
+        umma_commit(empty_bar(2 * qgp));  // G chunk free
         // ---- S_{g+1}
         if (g + 1 < nchunks) {
           const uint32_t gn = g + 1;
           const int lin = int(gn / C::NCH), cn = int(gn % C::NCH);
           if (cn == 0) wfull(2 * tok_kv_pair(lin), 0x908);
-          wfull(2 * tok_qg_pair(lin, cn), 0x909);
+          wfull(2 * tok_qg_pair(lin, cn) + 1, 0x909);
           wt(sd_free_da, g & 1, 0x90A);
           if (!ok) break;
           tc_fence_after();
@@ -810,12 +821,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         wt(e_full, g & 1, 0x90B);
         if (!ok) break;
         tc_fence_after();
+        {
+          const uint64_t dQm = sdesc(aQ, C::NC * 128, 1024);
 #pragma unroll
-        for (int k = 0; k < C::NC / 16; ++k)
-          umma_ss(tmem + C::U_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                  sdesc(aQ + k * 2048, C::NC * 128, 1024), idTD, (c == 0 && k == 0) ? 0u : 1u);
+          for (int k = 0; k < C::NC / 16; ++k)
+            umma_ss(tmem + C::U_COL, sdesc_add(dAB, kstep(k)), sdesc_add(dQm, k * 2048), idU,
+                    (c == 0 && k == 0) ? 0u : 1u);
+        }
         umma_commit(ab_free_e);
-        umma_commit(empty_bar(2 * qgp));  // Q chunk free
+        umma_commit(empty_bar(2 * qgp + 1));  // Q chunk free
         if (c == C::NCH - 1) umma_commit(acc_full);
       }
       umma_commit(drain);
