@@ -1107,19 +1107,28 @@ template <int D, int PS>
 struct QCfg {
   static constexpr int KV_TILE = T * D * 2;
   static constexpr int QB = PS * D * 2;
-  static constexpr int NSLOT = 5;  // K and V tiles alternate over 5 slots: 2.5 tiles of lookahead
+  // K(i) is read by S(i) and, a tile later, by dQ(i); V(i) only by dA(i).  So
+  // K gets three slots and V two: K(i+2) loads once dQ(i-1) is done and V(i+2)
+  // once dA(i) is, each about one tile before it is needed.
+  static constexpr int NK = 3, NV = 2;
+  static constexpr int NSLOT = NK + NV;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_G = QB;
-  static constexpr int OFF_RING = 2 * QB;
+  static constexpr int OFF_RING = 2 * QB;  // K slots 0..NK-1, then V slots
   static constexpr int OFF_COL = OFF_RING + NSLOT * KV_TILE;  // [2 bufs][lse2 | D][128] fp32
   static constexpr int OFF_BAR = OFF_COL + 2 * 2 * T * 4;
-  static constexpr int NBAR = 2 * NSLOT + 20;
-  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
-  static constexpr int SMEM = OFF_MISC + 16;
+  static constexpr int NBAR = 2 * NSLOT + 16;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // TMEM base, abort flag
+  static constexpr int OFF_FLAGS = OFF_MISC + 16;      // per K slot: control bits of the tile it holds
+  static constexpr int SMEM = OFF_FLAGS + 4 * NK;
   static constexpr int S_COL = 0, DA_COL = T, DS_COL = 2 * T, DQ_COL = 3 * T;  // dS: two buffers of T/2
   static constexpr int TMEM_COLS = tmem_cols_for(DQ_COL + D);
   static_assert(PS == 128 && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
 };
+
+// Per-tile control bits, written by the TMA producer next to the tile's K so
+// the UMMA issuer follows the tile sequence without walking it.
+enum : uint32_t { kNewHead = 1u, kHeadLast = 2u, kSegFirst = 4u, kSegLast = 8u };
 
 template <int D, int PS>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -1137,14 +1146,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sQ = sbase + C::OFF_Q, sG = sbase + C::OFF_G, sRing = sbase + C::OFF_RING;
   const uint32_t bar0 = sbase + C::OFF_BAR;
+  // slot s < NK holds K tiles, slot NK + j holds V tiles
   auto ring_full = [&](int s) { return bar0 + 8u * s; };
   auto ring_empty = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
+  auto k_slot = [](int li) { return li % C::NK; };
+  auto v_slot = [](int li) { return C::NK + li % C::NV; };
   const uint32_t b1 = bar0 + 8u * (2 * C::NSLOT);
-  const uint32_t q_full = b1, q_empty = b1 + 8, g_full = b1 + 16, g_empty = b1 + 24, s_full = b1 + 32,
-                 s_free = b1 + 40, da_full = b1 + 48, da_free = b1 + 56, ds_full = b1 + 64, ds_empty0 = b1 + 72,
-                 dq_empty = b1 + 88, col_full0 = b1 + 96, col_empty0 = b1 + 112, drain = b1 + 128;
+  const uint32_t q_full = b1, q_empty = b1 + 8, g_full = b1 + 16, g_empty = b1 + 24, sda_full = b1 + 32,
+                 sda_free = b1 + 40, ds_full = b1 + 48, ds_empty0 = b1 + 56, dq_empty = b1 + 72,
+                 col_full0 = b1 + 80, col_empty0 = b1 + 96, drain = b1 + 112;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+  uint32_t* tflags = reinterpret_cast<uint32_t*>(smem + C::OFF_FLAGS);
   float* cols = reinterpret_cast<float*>(smem + C::OFF_COL);
   const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
   const int64_t total = tph * a.H;
@@ -1161,10 +1174,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_empty, 1);
     mbar_init(g_full, 2);
     mbar_init(g_empty, 1);
-    mbar_init(s_full, 1);
-    mbar_init(s_free, kSoftWarps);
-    mbar_init(da_full, 1);
-    mbar_init(da_free, kSoftWarps);
+    mbar_init(sda_full, 1);
+    mbar_init(sda_free, kSoftWarps);
     mbar_init(ds_full, kSoftWarps);
     mbar_init(ds_empty0, 1);
     mbar_init(ds_empty0 + 8, 1);
@@ -1190,11 +1201,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmV);
       tma_prefetch_desc(&tmQ);
       TileWalker it(a, tb, te, T);
-      int hc = 0, prev_h = -1;
-      uint32_t e = 0;
+      int hc = 0, prev_h = -1, loaded = 0;
       bool ok = true;
       for (int li = 0; li < ntiles && ok; ++li) {
-        if (it.h != prev_h) {
+        const bool new_head = it.h != prev_h;
+        if (new_head) {
           if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0xC01);
           if (!ok) break;
           mbar_arrive_expect_tx(q_full, C::QB);
@@ -1203,115 +1214,109 @@ __global__ void __launch_bounds__(kThreads, 1)
           prev_h = it.h;
           ++hc;
         }
+        int64_t t0n;
+        int nn, hn;
+        it.peek_next(t0n, nn, hn);
+        const uint32_t fl = (new_head ? kNewHead : 0u) | ((li + 1 >= ntiles || hn != it.h) ? kHeadLast : 0u) |
+                            (it.seg_first ? kSegFirst : 0u) | (it.seg_last ? kSegLast : 0u);
 #pragma unroll
         for (int kv = 0; kv < 2; ++kv) {
-          const int s = int(e % C::NSLOT);
-          if (e >= uint32_t(C::NSLOT)) ok = mbar_wait(ring_empty(s), ((e / C::NSLOT) + 1) & 1, abort_flag, a.ws, 0xC02);
+          const int nsl = kv ? C::NV : C::NK, use = li / nsl;
+          const int s = kv ? v_slot(li) : k_slot(li);
+          if (use > 0) ok = mbar_wait(ring_empty(s), (use + 1) & 1, abort_flag, a.ws, 0xC02);
           if (!ok) break;
+          if (kv == 0) tflags[s] = fl;  // published by the arrive below
           mbar_arrive_expect_tx(ring_full(s), C::KV_TILE);
 #pragma unroll
           for (int dh = 0; dh < D / 64; ++dh)
             tma_load_3d(sRing + s * C::KV_TILE + dh * T * 128, kv ? &tmV : &tmK, ring_full(s), 64 * dh, it.h,
                         int(it.tok0));
-          ++e;
+          loaded = li + 1;
         }
         it.next();
       }
-      if (!ok) {
-        for (uint32_t k = (e > uint32_t(C::NSLOT) ? e - C::NSLOT : 0); k < e; ++k)
-          mbar_wait_bounded(ring_full(int(k % C::NSLOT)), (k / C::NSLOT) & 1, 200000000ull);
+      if (!ok) {  // let the copies in flight land before the CTA exits
+        for (int li = (loaded > C::NK ? loaded - C::NK : 0); li < loaded; ++li) {
+          mbar_wait_bounded(ring_full(k_slot(li)), (li / C::NK) & 1, 200000000ull);
+          if (li + C::NV >= loaded) mbar_wait_bounded(ring_full(v_slot(li)), (li / C::NV) & 1, 200000000ull);
+        }
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- UMMA issuer
+      // Order: S(0), dA(0);
+      // then per tile i: S(i+1), dA(i+1), dQ(i), so the next tile's scores are
+      // ready when the softmax warps finish tile i.  One commit announces S and
+      // dA together (the softmax warps read both at once); descriptors are
+      // built once per operand and stepped by constant offsets.
       constexpr uint32_t idPT = idesc_bf16(128, T, 0, 0);  // [proto x tok], K = d
       constexpr uint32_t idQ = idesc_bf16(128, D, 0, 1);   // [proto x d], K = tokens, A from TMEM
-      TileWalker cur(a, tb, te, T), nxt(a, tb, te, T), nx2(a, tb, te, T);
-      nxt.next();
-      nx2.next();
-      nx2.next();
+      const uint64_t dQs = sdesc(sQ, 16, 1024), dGs = sdesc(sG, 16, 1024);
+      auto step_p = [](int k) { return uint32_t((k >> 2) * (PS * 128) + (k & 3) * 32); };
+      auto step_t = [](int k) { return uint32_t((k >> 2) * (T * 128) + (k & 3) * 32); };
       int hc = 0, gc = 0, hp = 0;
       bool ok = true;
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
       };
-      auto issue_pt = [&](uint32_t dcol, uint32_t aop, uint32_t bop) {  // [proto x tok] = aop bop^T
-#pragma unroll
-        for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + dcol, sdesc(aop + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024),
-                  sdesc(bop + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024), idPT, k > 0 ? 1u : 0u);
+      // waits for tile li's K and V, returns its control bits
+      auto wait_kv = [&](int li) -> uint32_t {
+        wt(ring_full(k_slot(li)), (li / C::NK) & 1, 0xD02);
+        wt(ring_full(v_slot(li)), (li / C::NV) & 1, 0xD04);
+        return ok ? tflags[k_slot(li)] : 0u;
       };
-      // Issue order: S(0), dA(0); then per tile i: S(i+1), dA(i+1), dQ(i), so the
-      // next tile's scores are ready when the softmax warps finish tile i.
-      auto issue_dA = [&](int li, bool seg_first) -> bool {
-        const uint32_t eV = 2u * li + 1;
-        const int sV = int(eV % C::NSLOT);
-        if (seg_first) {
+      auto issue_sda = [&](int li, uint32_t fl) {
+        if (fl & kNewHead) {
+          wt(q_full, hc & 1, 0xD01);
+          ++hc;
+        }
+        if (fl & kSegFirst) {
           wt(g_full, gc & 1, 0xD03);
           ++gc;
         }
-        wt(ring_full(sV), (eV / C::NSLOT) & 1, 0xD04);
-        if (li > 0) wt(da_free, (li - 1) & 1, 0xD05);
-        if (!ok) return false;
+        if (!ok) return;
         tc_fence_after();
-        issue_pt(C::DA_COL, sG, sRing + sV * C::KV_TILE);
-        umma_commit(da_full);
-        umma_commit(ring_empty(sV));
-        return true;
+        const int sK = k_slot(li), sV = v_slot(li);
+        const uint64_t dK = sdesc(sRing + sK * C::KV_TILE, 16, 1024), dV = sdesc(sRing + sV * C::KV_TILE, 16, 1024);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          umma_ss(tmem + C::S_COL, sdesc_add(dQs, step_p(k)), sdesc_add(dK, step_t(k)), idPT, k > 0 ? 1u : 0u);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k)
+          umma_ss(tmem + C::DA_COL, sdesc_add(dGs, step_p(k)), sdesc_add(dV, step_t(k)), idPT, k > 0 ? 1u : 0u);
+        umma_commit(sda_full);
+        umma_commit(ring_empty(sV));                // V read by its only product
+        if (fl & kHeadLast) umma_commit(q_empty);   // last S of this head piece
+        if (fl & kSegLast) umma_commit(g_empty);    // last dA of this segment
       };
-      wt(q_full, 0, 0xD01);
-      wt(ring_full(0), 0, 0xD02);
-      if (ok) {
-        tc_fence_after();
-        issue_pt(C::S_COL, sQ, sRing);
-        umma_commit(s_full);
-        if (ntiles == 1 || nxt.h != cur.h) umma_commit(q_empty);
-        issue_dA(0, cur.seg_first);
-        if (cur.seg_last) umma_commit(g_empty);
-      }
-      bool first_of_hp = true;
+      uint32_t fl_cur = wait_kv(0);
+      if (ok) issue_sda(0, fl_cur);
       for (int li = 0; li < ntiles && ok; ++li) {
-        const uint32_t eK = 2u * li;
-        const int sK = int(eK % C::NSLOT);
-        const bool more = li + 1 < ntiles;
-        const bool newhead = more && nxt.h != cur.h;
-        if (more) {
-          // ---- S(i+1) = Q_r K(i+1)^T once the softmax warps hold S(i)
-          if (newhead) {
-            ++hc;
-            wt(q_full, hc & 1, 0xD06);
-          }
-          wt(s_free, li & 1, 0xD07);
-          wt(ring_full(int((eK + 2) % C::NSLOT)), ((eK + 2) / C::NSLOT) & 1, 0xD08);
+        uint32_t fl_next = 0;
+        if (li + 1 < ntiles) {
+          wt(sda_free, li & 1, 0xD07);  // the softmax warps hold S(i), dA(i)
+          fl_next = wait_kv(li + 1);
           if (!ok) break;
-          tc_fence_after();
-          issue_pt(C::S_COL, sQ, sRing + ((eK + 2) % C::NSLOT) * C::KV_TILE);
-          umma_commit(s_full);
-          if (li + 2 >= ntiles || nx2.h != nxt.h) umma_commit(q_empty);
-          // ---- dA(i+1) = G_r V(i+1)^T once they hold dA(i)
-          if (!issue_dA(li + 1, nxt.seg_first)) break;
-          if (nxt.seg_last) umma_commit(g_empty);
+          issue_sda(li + 1, fl_next);
+          if (!ok) break;
         }
         // ---- dQ += dS(i) K(i), dS read from TMEM
+        const bool first_of_hp = (fl_cur & kNewHead) != 0;
         wt(ds_full, li & 1, 0xD09);
         if (first_of_hp && hp > 0) wt(dq_empty, (hp - 1) & 1, 0xD0A);
         if (!ok) break;
         tc_fence_after();
         {
-          const uint32_t kaddr = sRing + sK * C::KV_TILE;
-          const uint32_t dsb = C::DS_COL + (li & 1) * (T / 2);
+          const int sK = k_slot(li);
+          const uint64_t dK = sdesc(sRing + sK * C::KV_TILE, T * 128, 1024);  // MN-major: d blocks 16 KB apart
+          const uint32_t dsb = tmem + C::DS_COL + (li & 1) * (T / 2);
 #pragma unroll
           for (int k = 0; k < T / 16; ++k)
-            umma_ts(tmem + C::DQ_COL, tmem + dsb + 8 * k, sdesc(kaddr + k * 2048, T * 128, 1024), idQ,
-                    (first_of_hp && k == 0) ? 0u : 1u);
+            umma_ts(tmem + C::DQ_COL, dsb + 8 * k, sdesc_add(dK, k * 2048), idQ, (first_of_hp && k == 0) ? 0u : 1u);
+          umma_commit(ds_empty0 + 8 * (li & 1));
+          umma_commit(ring_empty(sK));
         }
-        umma_commit(ds_empty0 + 8 * (li & 1));
-        umma_commit(ring_empty(sK));
-        const bool last_of_hp = !more || newhead;
-        if (last_of_hp) ++hp;
-        first_of_hp = last_of_hp;
-        cur.next();
-        nxt.next();
-        nx2.next();
+        if (fl_cur & kHeadLast) ++hp;
+        fl_cur = fl_next;
       }
       umma_commit(drain);
       mbar_wait_bounded(drain, 0, 200000000ull);
@@ -1371,8 +1376,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int li = 0; li < ntiles && ok; ++li) {
         const int buf = li & 1;
         ok = wwait(col_full0 + 8 * buf, (li >> 1) & 1, 0xF01);
-        if (ok) ok = wwait(s_full, li & 1, 0xF02);
-        if (ok) ok = wwait(da_full, li & 1, 0xF03);
+        if (ok) ok = wwait(sda_full, li & 1, 0xF02);
         // this tile's dS buffer was last read by dQ(i-2)
         if (ok && li > 1) ok = wwait(ds_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xF04);
         if (!ok) break;
@@ -1386,10 +1390,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) {  // the next tile's S and dA may now be written
-          mbar_arrive(s_free);
-          mbar_arrive(da_free);
-        }
+        if (lane == 0) mbar_arrive(sda_free);  // the next tile's S and dA may now be written
         // per-token values as 16-byte broadcasts: one shared-memory wavefront per 4 tokens
         const float4* cl4 = reinterpret_cast<const float4*>(cl);
 #pragma unroll
