@@ -625,14 +625,14 @@ struct TokCfg {
   static_assert(NC == T && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
 };
 
-// Slot pairs rotate roles so the next tile's K and V load two chunks before
-// the tile ends: tile li keeps K, V in pair (li & 1); its chunks alternate
-// between pair 1 - (li & 1) and pair 2; pair 1 - (li & 1) is free after the
-// next-to-last chunk and takes tile li+1's K and V.  A chunk pair holds G in
-// its first slot and Q in the second, so the four 64-column blocks of G and Q
-// sit at one stride and [G | Q] is a single N = 2D operand.
-__device__ __forceinline__ int tok_kv_pair(int li) { return li & 1; }
-__device__ __forceinline__ int tok_qg_pair(int li, int c) { return (c & 1) ? 2 : 1 - (li & 1); }
+// Pair 0 holds the tile's K and V; the next tile's K loads into it once the
+// tile's last S has read K, its V once the last dA has read V, and both tiles
+// are pulled into L2 a tile ahead.  Chunks alternate between pairs 1 and 2
+// (the chunk count per tile is even).  A chunk pair holds G in its first slot
+// and Q in the second, so the four 64-column blocks of G and Q sit at one
+// stride and [G | Q] is a single N = 2D operand.
+__device__ __forceinline__ int tok_kv_pair(int) { return 0; }
+__device__ __forceinline__ int tok_qg_pair(int, int c) { return 1 + (c & 1); }
 
 template <int D, int P>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -705,6 +705,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmG);
       TileWalker it(a, tb, te, T), nx(a, tb, te, T);
       nx.next();
+      static_assert(C::NCH % 2 == 0, "chunks alternate between two pairs");
       int uses[C::NSLOT] = {0, 0, 0, 0, 0, 0};
       bool ok = true;
       // box origin (64*dh, c1, c2): K / V maps are (d, head, token); Q / G maps
@@ -717,21 +718,29 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(slot_addr(s) + dh * T * 128, map, full_bar(s), 64 * dh, c1, c2);
       };
-      auto load_kv = [&](int li, const TileWalker& w) {
-        const int pr = tok_kv_pair(li);
-        load(2 * pr, &tmK, w.h, int(w.tok0));
-        load(2 * pr + 1, &tmV, w.h, int(w.tok0));
+      auto prefetch_kv = [&](const TileWalker& w) {
+#pragma unroll
+        for (int dh = 0; dh < D / 64; ++dh) {
+          tma_prefetch_l2_3d(&tmK, 64 * dh, w.h, int(w.tok0));
+          tma_prefetch_l2_3d(&tmV, 64 * dh, w.h, int(w.tok0));
+        }
       };
-      load_kv(0, it);
+      // Order of loads: ..., Q/G(li, last), K(li+1), Q/G(li+1, 0), V(li+1), ...:
+      // K(li+1) waits for S(li, last), V(li+1) for dA(li, last).
+      load(0, &tmK, it.h, int(it.tok0));
+      load(1, &tmV, it.h, int(it.tok0));
+      if (ntiles > 1) prefetch_kv(nx);
       for (int li = 0; li < ntiles && ok; ++li) {
         for (int c = 0; c < C::NCH && ok; ++c) {
           const int pr = tok_qg_pair(li, c);
           load(2 * pr + 1, &tmQ, c * C::NC, it.h);
           load(2 * pr, &tmG, c * C::NC, int(it.b) * a.H + it.h);
-          if (c == C::NCH - 1 && li + 1 < ntiles) load_kv(li + 1, nx);
+          if (c == 0 && li > 0) load(1, &tmV, it.h, int(it.tok0));
+          if (c == C::NCH - 1 && li + 1 < ntiles) load(0, &tmK, nx.h, int(nx.tok0));
         }
         it.next();
         nx.next();
+        if (li + 2 < ntiles) prefetch_kv(nx);
       }
       if (!ok) {
         for (int s = 0; s < C::NSLOT; ++s)
