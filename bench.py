@@ -272,7 +272,8 @@ def run_ours(args, spec, lens):
         else:
             ach, peak, unit, bound = work.bytes / per_call_s / 1e9, pk["hbm_gbs"], "GB/s", "hbm"
         return {"kernel": name, "bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
-                "traffic": traffic_for(name), "avg_launch_ms": kms / kn, "launches": kn,
+                "traffic": traffic_for(name), "traffic_per": "call (DRAM bytes, ncu, scaled from a sub-batch)",
+                "avg_launch_ms": kms / kn, "launches": kn,
                 "launches_per_call": kn // calls, "ms_per_call": kms / calls,
                 "peak_source": f"{pk['source']} ({'bf16 sustained' if unit == 'TFLOP/s' else 'HBM copy'})",
                 "algorithmic_per_call": work.flops if unit == "TFLOP/s" else work.bytes}
@@ -305,7 +306,8 @@ def run_ours(args, spec, lens):
 
 
 def traffic_for(kernel_name):
-    """DRAM bytes per launch from the committed ncu summary, if it matches the
+    """DRAM bytes per call of the kernel (for the split backward: its token-side
+    and dQ kernels together) from the committed ncu summary, if it matches the
     kernel source that is built now; else None."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
@@ -319,7 +321,7 @@ def traffic_for(kernel_name):
         return None
     from paper_2609_08443_gb300 import build
 
-    return ent.get("bytes_per_launch") if ent.get("source_hash") == build.source_hash() else None
+    return ent.get("bytes_per_call") if ent.get("source_hash") == build.source_hash() else None
 
 
 def e2e_run(args, spec, dev):
