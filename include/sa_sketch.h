@@ -151,8 +151,11 @@ uint64_t sa_launch_count(void);
 
 /* Kernel selection for all later calls in this process: 0 (default) lets each
  * call pick the tensor-core kernels where its shape is supported, 1 forces the
- * CUDA-core kernels everywhere (a cross-check of the two).  The workspace size
- * depends on the selection: size it after choosing. */
+ * CUDA-core kernels everywhere (a cross-check of the two), 2 keeps the
+ * tensor cores but runs the forward for P = 512 (and P = 256 with d = 128) as a
+ * per-token lse pass followed by prototype slices instead of the cluster-pair
+ * kernel (another cross-check).  The workspace size depends on the selection:
+ * size it after choosing. */
 sa_status sa_select_path(int path);
 
 /* Name of the kernel that a forward (bwd = 0) or backward (bwd = 1) call with

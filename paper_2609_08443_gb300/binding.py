@@ -125,7 +125,8 @@ def sa_launch_count() -> int:
 
 
 def sa_select_path(path: int) -> None:
-    """0: tensor-core kernels where supported (default); 1: CUDA cores only."""
+    """0: tensor-core kernels where supported (default); 1: CUDA cores only;
+    2: tensor cores with the lse pass + prototype slices for P = 512."""
     _check(load().sa_select_path(int(path)), "sa_select_path")
 
 

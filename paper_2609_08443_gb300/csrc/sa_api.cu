@@ -15,7 +15,7 @@
 
 namespace {
 
-std::atomic<int> g_path{0};  // 0 = choose per shape, 1 = CUDA cores only
+std::atomic<int> g_path{0};  // 0 = choose per shape, 1 = CUDA cores only, 2 = lse pass + slices
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -161,7 +161,8 @@ sa::Args make_args(const void* K, const void* V, const int32_t* cu, int B, int64
 // ------------------------------------------------------- tensor-core helpers
 namespace sa {
 
-bool tc_path_enabled() { return g_path.load() == 0; }
+bool tc_path_enabled() { return g_path.load() != 1; }
+bool tc_fwd_sliced_selected() { return g_path.load() == 2; }
 
 namespace tcc {
 
@@ -353,7 +354,7 @@ sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches)
 uint64_t sa_launch_count(void) { return g_launches.load(); }
 
 sa_status sa_select_path(int path) {
-  if (path != 0 && path != 1) return SA_ERR_INVALID_ARG;
+  if (path < 0 || path > 2) return SA_ERR_INVALID_ARG;
   g_path.store(path);
   return SA_OK;
 }

@@ -68,6 +68,83 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 
+// ------------------------------------------------------------ CTA clusters
+// Rank of this CTA in its cluster, the shared::cluster address of the same
+// shared-memory offset in CTA `rank`, and the cluster-scope forms of the
+// mbarrier operations used when two CTAs exchange per-token statistics.
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+// arrive (release at cluster scope) on an mbarrier of this CTA or of a peer;
+// `bar_cl` is a shared::cluster address (from mapa_shared)
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cl) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cl) : "memory");
+}
+// arrive without ordering prior memory operations (the peer only learns that
+// values this thread already consumed may be overwritten)
+__device__ __forceinline__ void mbar_arrive_relaxed_cluster(uint32_t bar_cl) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cl) : "memory");
+}
+// 8-byte store into a peer's shared memory that completes `bytes` of the
+// transaction count of the peer's mbarrier `bar_cl` (no release fence needed:
+// the data is visible to whoever observes that barrier phase complete)
+__device__ __forceinline__ void st_async_f2(uint32_t dst_cl, float2 v, uint32_t bar_cl) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(dst_cl),
+               "f"(v.x), "f"(v.y), "r"(bar_cl)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ float2 ld_cluster_f2(uint32_t addr_cl) {
+  float2 v;
+  asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr_cl) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_cluster_u32(uint32_t addr_cl) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(addr_cl) : "memory");
+  return v;
+}
+// Every thread of every CTA of the cluster must execute this (all CTAs of a
+// cluster are resident together, so it completes once all have arrived).
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Bounded wait with acquire at cluster scope (peers' writes become visible).
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, volatile int* abort_flag, void* ws,
+                                                  uint32_t site) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if ((it & 63u) == 0u) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        ws_set_error(ws, SA_ERR_TIMEOUT, site);
+        return false;
+      }
+    }
+  }
+}
+
 // ----------------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const void* tmap) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
@@ -211,6 +288,78 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// ------------------------------------------- per-thread softmax arithmetic
+// Three-input maximum (one instruction on sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// max of v[0..N) with four independent chains (N a multiple of 8)
+template <int N>
+__device__ __forceinline__ float row_max(const float* v) {
+  static_assert(N % 8 == 0, "row_max works on multiples of 8 values");
+  float a0 = fmaxf(v[0], v[1]), a1 = fmaxf(v[2], v[3]), a2 = fmaxf(v[4], v[5]), a3 = fmaxf(v[6], v[7]);
+#pragma unroll
+  for (int j = 8; j < N; j += 8) {
+    a0 = fmax3(a0, v[j], v[j + 1]);
+    a1 = fmax3(a1, v[j + 2], v[j + 3]);
+    a2 = fmax3(a2, v[j + 4], v[j + 5]);
+    a3 = fmax3(a3, v[j + 6], v[j + 7]);
+  }
+  return fmaxf(fmax3(a0, a1, a2), a3);
+}
+
+// v[j] <- 2^(v[j] * c2 - sh) (one fused multiply-add per value, two values per
+// instruction); returns the sum of the results, accumulated in four chains.
+template <int N>
+__device__ __forceinline__ float exp2_shift_sum(float* v, float c2, float sh) {
+  static_assert(N % 4 == 0, "exp2_shift_sum works on multiples of 4 values");
+  const float2 cc = make_float2(c2, c2), ns = make_float2(-sh, -sh);
+  float2 z0 = make_float2(0.f, 0.f), z1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int j = 0; j < N; j += 4) {
+    float2 x0 = __ffma2_rn(make_float2(v[j], v[j + 1]), cc, ns);
+    float2 x1 = __ffma2_rn(make_float2(v[j + 2], v[j + 3]), cc, ns);
+    x0.x = ex2(x0.x);
+    x0.y = ex2(x0.y);
+    x1.x = ex2(x1.x);
+    x1.y = ex2(x1.y);
+    v[j] = x0.x;
+    v[j + 1] = x0.y;
+    v[j + 2] = x1.x;
+    v[j + 3] = x1.y;
+    z0 = __fadd2_rn(z0, x0);
+    z1 = __fadd2_rn(z1, x1);
+  }
+  return (z0.x + z0.y) + (z1.x + z1.y);
+}
+
+// v[j] <- 2^(v[j] * c2 - sh), no sum (sh = +inf gives exact zeros)
+template <int N>
+__device__ __forceinline__ void exp2_shift(float* v, float c2, float sh) {
+  const float2 cc = make_float2(c2, c2), ns = make_float2(-sh, -sh);
+#pragma unroll
+  for (int j = 0; j < N; j += 2) {
+    float2 x = __ffma2_rn(make_float2(v[j], v[j + 1]), cc, ns);
+    v[j] = ex2(x.x);
+    v[j + 1] = ex2(x.y);
+  }
+}
+
+// v[j] <- v[j] * f, two values per instruction
+template <int N>
+__device__ __forceinline__ void scale_row(float* v, float f) {
+  const float2 ff = make_float2(f, f);
+#pragma unroll
+  for (int j = 0; j < N; j += 2) {
+    const float2 x = __fmul2_rn(make_float2(v[j], v[j + 1]), ff);
+    v[j] = x.x;
+    v[j + 1] = x.y;
+  }
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {

@@ -7,6 +7,7 @@ namespace sa {
 bool tc_fwd_supported(int P, int d, sa_dtype dt);
 bool tc_fwd_needs_lse_pass_d(int P, int d);  // lse pass, then 256-prototype slices
 bool tc_path_enabled();
+bool tc_fwd_sliced_selected();  // sa_select_path(2)
 bool tc_bwd_supported(int P, int d, sa_dtype dt);
 const char* tc_fwd_name(int P, int d);
 const char* tc_bwd_name(int P, int d);

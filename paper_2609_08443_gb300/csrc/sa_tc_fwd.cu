@@ -17,6 +17,14 @@
 //      N = d) or  O^T = V^T A^T  (d = 128: M = d, N = prototypes).
 //   5. When a user's segment ends the sketch (or a worker's piece of it) is
 //      read back from TMEM and stored.
+// Pair mode (P = 512): a cluster of two CTAs shares each tile; CTA r holds
+// prototypes [256 r, 256 r + 256).  Per token, warpgroup 1 hands its (max,
+// sum) to warpgroup 0 through shared memory; warpgroup 0 combines the CTA's
+// two partials, pushes the result into the peer CTA's shared memory with
+// st.async (whose completion is counted on the peer's mbarrier, so no
+// cluster-scope fence is needed), combines its own and the peer's value in
+// CTA order -- bitwise the same (max, sum) in both CTAs -- and hands the final
+// pair back to warpgroup 1.
 // Warp roles: 0 = TMA producer, 1 = UMMA issuer, 2 = TMEM allocator,
 // 4..11 = softmax + epilogue.  Every wait is bounded (sa_ptx.cuh).
 #include <cuda.h>
@@ -33,7 +41,7 @@ namespace tcf {
 using namespace ptx;
 using namespace tcc;
 
-enum Mode { kFused = 0, kSliced = 1 };
+enum Mode { kFused = 0, kSliced = 1, kPair = 2 };
 
 template <int D, int PS, int MODE>
 struct Cfg {
@@ -41,15 +49,16 @@ struct Cfg {
   static constexpr int Q_BYTES = PS * D * 2;
   static constexpr int W_BYTES = T * PS * 2;
   static constexpr int NSLOT = (D == 128) ? 3 : 6;
-  static constexpr int STATS = (MODE == kFused) ? 2 * T * 8 : 0;
+  static constexpr int STATS = (MODE == kSliced) ? 0 : 2 * T * 8;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_RING = OFF_Q + Q_BYTES;
   static constexpr int OFF_W = OFF_RING + NSLOT * KV_TILE;
   static constexpr int OFF_STATS = OFF_W + W_BYTES;
   static constexpr int OFF_BAR = OFF_STATS + STATS;
-  static constexpr int NBAR = 2 * NSLOT + 12;
-  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // tmem address, abort flag
+  static constexpr int NBAR = 2 * NSLOT + 13;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // tmem address, abort flag, skip flag (pair)
   static constexpr int SMEM = OFF_MISC + 16;
+  static_assert(SMEM <= 232448, "shared memory budget");
   static constexpr bool TRANS = (D == 128);  // O^T = V^T A^T
   static constexpr int O_COLS = TRANS ? PS : (PS / 128) * D;
   static constexpr int S_COL = 0;
@@ -66,11 +75,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   using C = Cfg<D, PS, MODE>;
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (ws_failed(a.ws)) return;
+  constexpr bool PAIR = (MODE == kPair);
+  // A pair's CTAs must both reach the cluster barriers below, so pair mode
+  // never returns early: a failed call or a misaligned base only skips work.
+  bool skip = ws_failed(a.ws);
   if (smem_u32(smem) & 1023u) {  // 128-byte swizzle atoms need 1024-byte alignment
     if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xA11u);
-    return;
+    skip = true;
   }
+  if (!PAIR && skip) return;
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sQ = sbase + C::OFF_Q, sRing = sbase + C::OFF_RING, sW = sbase + C::OFF_W;
   const uint32_t bar0 = sbase + C::OFF_BAR;
@@ -78,16 +91,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto ring_empty = [&](int s) { return bar0 + 8u * (C::NSLOT + s); };
   const uint32_t q_full = bar0 + 8u * (2 * C::NSLOT + 0), q_empty = q_full + 8, s_full = q_full + 16,
                  s_empty = q_full + 24, w_full = q_full + 32, w_empty = q_full + 40, o_full = q_full + 48,
-                 o_empty = q_full + 56, drain = q_full + 64, st_ready = q_full + 72, st_used = q_full + 80;
+                 o_empty = q_full + 56, drain = q_full + 64, st_ready = q_full + 72, st_used = q_full + 80,
+                 r_full = q_full + 88, r_used = q_full + 96;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+  volatile uint32_t* skip_flag = reinterpret_cast<volatile uint32_t*>(smem + C::OFF_MISC + 8);
+  const uint32_t rank = PAIR ? cluster_rank() : 0u, peer = rank ^ 1u;
 
   const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
   const int64_t total = tph * a.H;
-  const int W = gridDim.x, wk = blockIdx.x, slice = blockIdx.y;
+  // pair mode: the two CTAs of cluster c are worker c; CTA rank r is slice r
+  const int W = PAIR ? int(gridDim.x >> 1) : int(gridDim.x);
+  const int wk = PAIR ? int(blockIdx.x >> 1) : int(blockIdx.x);
+  const int slice = PAIR ? int(rank) : int(blockIdx.y);
   const int p0 = slice * PS;
   const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
-  const int ntiles = int(te - tb);
+  int ntiles = int(te - tb);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::NSLOT; ++s) {
@@ -103,14 +122,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(o_full, 1);
     mbar_init(o_empty, kSoftWarps);
     mbar_init(drain, 1);
-    mbar_init(st_ready, kSoftWarps);
-    mbar_init(st_used, kSoftWarps);
+    // pair mode: st_ready = warpgroup 1's partials are in, st_used = the final
+    // pair is in (each 4 warps); r_full = the peer's pair has landed (one local
+    // expect_tx + 1 KB of st.async), r_used = the peer has read what this CTA
+    // pushed (the peer's 4 warps of warpgroup 0)
+    mbar_init(st_ready, PAIR ? kSoftWarps / 2 : kSoftWarps);
+    mbar_init(st_used, PAIR ? kSoftWarps / 2 : kSoftWarps);
+    mbar_init(r_full, 1);
+    mbar_init(r_used, kSoftWarps / 2);
     *abort_flag = 0;
+    *skip_flag = skip ? 1u : 0u;
     fence_mbar_init();
   }
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
   tc_fence_before();
-  __syncthreads();
+  if (PAIR) {
+    // barriers of both CTAs initialised; both CTAs skip if either must
+    cluster_sync_all();
+    if (*skip_flag || ld_cluster_u32(mapa_shared(smem_u32(smem + C::OFF_MISC + 8), peer))) ntiles = 0;
+  } else {
+    __syncthreads();
+  }
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
@@ -120,11 +152,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
       tma_prefetch_desc(&tmQ);
-      TileWalker it(a, tb, te, T), pv(a, tb, te, T);
+      TileWalker it(a, tb, te, T), pv(a, tb, te, T), pf(a, tb, te, T);
+      pf.next();
+      pf.next();
       int hc = 0, prev_h = -1;
       uint32_t e = 0;
       bool ok = true;
       for (int li = 0; li <= ntiles && ok; ++li) {
+        if (li + 2 < ntiles) {
+          // K and V of tile li + 2 into L2, so the ring loads hit L2
+#pragma unroll
+          for (int dh = 0; dh < D / 64; ++dh) {
+            tma_prefetch_l2_3d(&tmK, 64 * dh, pf.h, int(pf.tok0));
+            tma_prefetch_l2_3d(&tmV, 64 * dh, pf.h, int(pf.tok0));
+          }
+          pf.next();
+        }
         if (li < ntiles) {
           if (it.h != prev_h) {
             if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0x101);
@@ -272,6 +315,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
       };
+      // pair mode: the peer's R buffer (second half of the stats area) and
+      // its barriers, as shared::cluster addresses
+      const uint32_t r_peer = PAIR ? mapa_shared(sbase + C::OFF_STATS + 8u * T, peer) : 0u;
+      const uint32_t r_full_peer = PAIR ? mapa_shared(r_full, peer) : 0u;
+      const uint32_t r_used_peer = PAIR ? mapa_shared(r_used, peer) : 0u;
+      // (max, sum) of two disjoint prototype sets, a before b
+      auto combine = [&](float2 x, float2 y) {
+        const float M = fmaxf(x.x, y.x);
+        return make_float2(M, x.y * ex2((x.x - M) * c2) + y.y * ex2((y.x - M) * c2));
+      };
       for (int li = 0; li < ntiles && ok; ++li) {
         float lse_nxt = 0.f;
         if (MODE == kSliced) {  // next tile's lse, issued before this tile's scores are live
@@ -292,45 +345,68 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(s_empty);
         const bool valid = row < cur.n;
         const int64_t tok = cur.tok0 + row;
-        if (MODE == kFused) {
-          float m = v[0];
-#pragma unroll
-          for (int j = 1; j < C::HALF; ++j) m = fmaxf(m, v[j]);
-          const float mc = m * c2;
-          float z = 0.f;
-#pragma unroll
-          for (int j = 0; j < C::HALF; ++j) {
-            v[j] = ex2(fmaf(v[j], c2, -mc));
-            z += v[j];
-          }
-          // exchange (max, sum) with the other warpgroup's thread of this token
-          if (li > 0) {
-            ok = wwait(st_used, (li - 1) & 1, 0x304);
+        if (MODE == kFused || MODE == kPair) {
+          const float m = row_max<C::HALF>(v);
+          const float z = exp2_shift_sum<C::HALF>(v, c2, m * c2);
+          float M, Z, f;
+          if (PAIR) {
+            // stats[0..T) = L: warpgroup 1's partial, then the final pair;
+            // stats[T..2T) = R: the peer CTA's combined pair (st.async)
+            float2 fin;
+            if (sw == 1) {
+              stats[row] = make_float2(m, z);
+              __syncwarp();
+              if (lane == 0) mbar_arrive(st_ready);
+              ok = wwait(st_used, li & 1, 0x306);
+              if (!ok) break;
+              fin = stats[row];
+            } else {
+              ok = wwait(st_ready, li & 1, 0x305);
+              if (!ok) break;
+              const float2 loc = combine(make_float2(m, z), stats[row]);
+              if (li > 0) {
+                ok = wwait(r_used, (li - 1) & 1, 0x307);  // the peer has read the last push
+                if (!ok) break;
+              }
+              if (warp == kSoftWarp0 && lane == 0) mbar_arrive_expect_tx(r_full, 8u * T);
+              st_async_f2(r_peer + 8u * row, loc, r_full_peer);
+              ok = wwait(r_full, li & 1, 0x308);
+              if (!ok) break;
+              const float2 oth = stats[T + row];
+              __syncwarp();
+              if (lane == 0) mbar_arrive_relaxed_cluster(r_used_peer);
+              fin = rank == 0 ? combine(loc, oth) : combine(oth, loc);
+              stats[row] = fin;
+              __syncwarp();
+              if (lane == 0) mbar_arrive(st_used);
+            }
+            M = fin.x;
+            Z = fin.y;
+            f = ex2((m - M) * c2) / Z;
+          } else {
+            // exchange (max, sum) with the other warpgroup's thread of this token
+            if (li > 0) {
+              ok = wwait(st_used, (li - 1) & 1, 0x304);
+              if (!ok) break;
+            }
+            stats[sw * T + row] = make_float2(m, z);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(st_ready);
+            ok = wwait(st_ready, li & 1, 0x305);
             if (!ok) break;
+            const float2 o = stats[(1 - sw) * T + row];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(st_used);
+            M = fmaxf(m, o.x);
+            const float f_self = ex2((m - M) * c2), f_other = ex2((o.x - M) * c2);
+            Z = z * f_self + o.y * f_other;
+            f = f_self / Z;
           }
-          stats[sw * T + row] = make_float2(m, z);
-          __syncwarp();
-          if (lane == 0) mbar_arrive(st_ready);
-          ok = wwait(st_ready, li & 1, 0x305);
-          if (!ok) break;
-          const float2 o = stats[(1 - sw) * T + row];
-          __syncwarp();
-          if (lane == 0) mbar_arrive(st_used);
-          const float M = fmaxf(m, o.x);
-          const float f_self = ex2((m - M) * c2), f_other = ex2((o.x - M) * c2);
-          const float Z = z * f_self + o.y * f_other;
-          const float f = f_self / Z;
-#pragma unroll
-          for (int j = 0; j < C::HALF; ++j) v[j] *= f;
-          if (sw == 0 && valid && lse_out) lse_out[tok * a.H + cur.h] = M * a.scale + logf(Z);
+          // rows past the tile's tokens get exact zero weights
+          scale_row<C::HALF>(v, valid ? f : 0.f);
+          if (rank == 0 && sw == 0 && valid && lse_out) lse_out[tok * a.H + cur.h] = M * a.scale + logf(Z);
         } else {
-          const float L2 = lse_cur * 1.4426950408889634f;
-#pragma unroll
-          for (int j = 0; j < C::HALF; ++j) v[j] = ex2(fmaf(v[j], c2, -L2));
-        }
-        if (!valid) {
-#pragma unroll
-          for (int j = 0; j < C::HALF; ++j) v[j] = 0.f;
+          exp2_shift<C::HALF>(v, c2, valid ? lse_cur * 1.4426950408889634f : INFINITY);
         }
         if (li > 0) {
           ok = wwait(w_empty, (li - 1) & 1, 0x302);
@@ -375,6 +451,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
+  // the peer may still read this CTA's statistics or arrive on its barriers
+  if (PAIR) cluster_sync_all();
 }
 
 // ------------------------------------------------------------------ lse only
@@ -595,6 +673,22 @@ static cudaError_t launch_fwd_t(const Args& a, int W, float* sketch, float* lse_
   auto fn = &tc_fwd_kernel<D, PS, MODE>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
+  if (MODE == kPair) {
+    // one cluster of two CTAs per worker; CTA rank r holds prototypes [PS r, PS r + PS)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * W, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = C::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, fn, tk, tv, tq, a, sketch, lse_out, lse_in);
+  }
   dim3 grid(W, a.P / PS);
   fn<<<grid, kThreads, C::SMEM, st>>>(tk, tv, tq, a, sketch, lse_out, lse_in);
   return cudaGetLastError();
@@ -623,13 +717,17 @@ bool tc_fwd_supported(int P, int d, sa_dtype dt) {
   return tcc::device_is_sm103() && tc_path_enabled();
 }
 
-// P = 512, or P = 256 with d = 128 (whose fused variant does not fit 227 KB of
-// shared memory next to the statistics exchange): lse pass, then slices of 256.
-bool tc_fwd_needs_lse_pass_d(int P, int d) { return P == 512 || (P == 256 && d == 128); }
+// By default every supported shape normalises inside the forward kernel:
+// P <= 256 in one CTA, P = 512 in a cluster pair.  Path 2 of sa_select_path
+// runs P = 512 (and P = 256 with d = 128) as a per-token lse pass followed by
+// 256-prototype slices that take that lse -- the same result computed another
+// way, kept as a cross-check.
+bool tc_fwd_needs_lse_pass_d(int P, int d) { return tc_fwd_sliced_selected() && (P == 512 || (P == 256 && d == 128)); }
 
 const char* tc_fwd_name(int P, int d) {
   if (tc_fwd_needs_lse_pass_d(P, d)) return d == 128 ? "tc_fwd_kernel<128,256,sliced>" : "tc_fwd_kernel<64,256,sliced>";
-  if (P == 256) return "tc_fwd_kernel<64,256,fused>";
+  if (P == 512) return d == 128 ? "tc_fwd_kernel<128,256,pair>" : "tc_fwd_kernel<64,256,pair>";
+  if (P == 256) return d == 128 ? "tc_fwd_kernel<128,256,fused>" : "tc_fwd_kernel<64,256,fused>";
   return d == 128 ? "tc_fwd_kernel<128,128,fused>" : "tc_fwd_kernel<64,128,fused>";
 }
 
@@ -662,7 +760,12 @@ cudaError_t launch_tc_fwd(const Args& a, int W, float* sketch, float* lse, cudaS
   if (tc_fwd_needs_lse_pass_d(a.P, a.d))  // lse (from launch_tc_lse beforehand) is an input here
     return a.d == 128 ? launch_fwd_t<128, 256, kSliced>(a, W, sketch, nullptr, lse, st)
                       : launch_fwd_t<64, 256, kSliced>(a, W, sketch, nullptr, lse, st);
-  if (a.P == 256) return launch_fwd_t<64, 256, kFused>(a, W, sketch, lse, nullptr, st);
+  if (a.P == 512)
+    return a.d == 128 ? launch_fwd_t<128, 256, kPair>(a, W, sketch, lse, nullptr, st)
+                      : launch_fwd_t<64, 256, kPair>(a, W, sketch, lse, nullptr, st);
+  if (a.P == 256)
+    return a.d == 128 ? launch_fwd_t<128, 256, kFused>(a, W, sketch, lse, nullptr, st)
+                      : launch_fwd_t<64, 256, kFused>(a, W, sketch, lse, nullptr, st);
   return a.d == 128 ? launch_fwd_t<128, 128, kFused>(a, W, sketch, lse, nullptr, st)
                     : launch_fwd_t<64, 128, kFused>(a, W, sketch, lse, nullptr, st);
 }

@@ -31,3 +31,22 @@ def test_tensor_core_path_matches_cuda_core_path(cuda_lib, P, d):
 
 def test_fp32_uses_cuda_cores(cuda_lib):
     assert binding.sa_main_kernel_name(64, 64, binding.SA_F32, False).startswith("simt")
+
+
+@pytest.mark.parametrize("P,d", [(512, 128), (512, 64), (256, 128)])
+def test_pair_forward_matches_lse_pass_and_slices(cuda_lib, P, d):
+    """The cluster-pair forward (one kernel, per-token statistics exchanged
+    between two CTAs) against the lse pass + prototype slices (two kernels)."""
+    spec = wl.custom([700, 0, 128, 129, 3000, 1], H=2, P=P, d=d, dtype=wl.BF16, seed=P + 3 * d)
+    host = wl.make_host(spec)
+    t = wl.host_to_torch(spec, host, torch.device("cuda"))
+    fused = harness.gpu_outputs(spec, t, bwd=False)
+    binding.sa_select_path(2)
+    try:
+        assert "sliced" in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
+        sliced = harness.gpu_outputs(spec, t, bwd=False)
+    finally:
+        binding.sa_select_path(0)
+    assert "sliced" not in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
+    assert harness.rel_err(fused["sketch"], sliced["sketch"]) <= 2e-2
+    assert abs(fused["lse"] - sliced["lse"]).max() <= 5e-3 * max(1.0, abs(sliced["lse"]).max())
