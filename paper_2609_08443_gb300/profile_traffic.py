@@ -38,7 +38,7 @@ def kernel_bytes(report: str) -> dict:
             continue
         name = r[i_name].split("(")[0].replace("void ", "").split("::")[-1].replace(" ", "")
         if name.startswith("tc_fwd_kernel<"):  # the library names the forward's mode
-            name = name[: name.rfind(",") + 1] + {"0>": "fused>", "1>": "sliced>"}.get(name[name.rfind(",") + 1:], "?>")
+            name = name[: name.rfind(",") + 1] + {"0>": "fused>", "1>": "sliced>", "2>": "pair>"}.get(name[name.rfind(",") + 1:], "?>")
         b = sum(float(r[c].replace(",", "")) * _UNITS[units[c]] for c in cols)
         e = agg.setdefault(name, {"bytes": 0.0, "launches": 0})
         e["bytes"] += b
