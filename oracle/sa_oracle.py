@@ -30,6 +30,12 @@ is the chain rule of the three forward steps with upstream G = dL/dO[b, h]:
     dQ[h] += scale * dS K_b    summed over ALL users, because the prototypes are
                                shared globally (Sec. 3.1)
 
+Stacked refinement (Sec. 3.3): from the second SA step on, the queries are the
+user's own refined sketch times W_Q^(l), so every user b has its own
+prototypes Q[b, h] ([B, H, P, d]); the three steps are otherwise unchanged and
+dQ[b, h] = scale * dS K_b collects only user b's tokens
+(``sa_forward_per_user`` / ``sa_backward_per_user``).
+
 All arithmetic is float64; bf16 inputs arrive already widened exactly.
 Parity pins for both functions live in ``tests/test_oracle.py`` (brute force
 in 50-digit arithmetic, closed forms, invariants, finite differences).
@@ -108,3 +114,51 @@ def sa_backward(K, V, cu_seqlens, Q, scale, dO):
             dK[t0:t1, h, :] = scale * (dS.T @ Q[h])
             dQ[h] += scale * (dS @ Kb)
     return dK, dV, dQ
+
+
+def sa_forward_per_user(K, V, cu_seqlens, Qu, scale, with_lse=False):
+    """Sketch with per-user queries (Sec. 3.3, S^(l) = (X~^(l) W_Q^(l)) (X W_K^(l))^T / sqrt(d)):
+    Qu[b, h] ([B, H, P, d]) replaces Q[h] for user b; everything else as ``sa_forward``."""
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Qu = np.asarray(Qu, dtype=np.float64)
+    B, H, P, d = Qu.shape
+    sl = _user_slices(cu_seqlens)
+    assert len(sl) == B
+    O = np.zeros((B, H, P, d))
+    lse = np.zeros((K.shape[0], H))
+    for b, (t0, t1) in enumerate(sl):
+        if t1 == t0:
+            continue
+        for h in range(H):
+            S = affinity(Qu[b, h], K[t0:t1, h, :], scale)
+            O[b, h] = proto_softmax(S) @ V[t0:t1, h, :]
+            if with_lse:
+                m = S.max(axis=0)
+                lse[t0:t1, h] = m + np.log(np.exp(S - m).sum(axis=0))
+    return (O, lse) if with_lse else O
+
+
+def sa_backward_per_user(K, V, cu_seqlens, Qu, scale, dO):
+    """Gradients (dK [N,H,d], dV [N,H,d], dQu [B,H,P,d]) of L = sum(dO * O) with
+    per-user queries: dQu[b, h] = scale * dS K_b holds only user b's tokens."""
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Qu = np.asarray(Qu, dtype=np.float64)
+    dO = np.asarray(dO, dtype=np.float64)
+    B, H, P, d = Qu.shape
+    dK = np.zeros_like(K)
+    dV = np.zeros_like(V)
+    dQu = np.zeros_like(Qu)
+    for b, (t0, t1) in enumerate(_user_slices(cu_seqlens)):
+        if t1 == t0:
+            continue
+        for h in range(H):
+            Kb, Vb, G = K[t0:t1, h, :], V[t0:t1, h, :], dO[b, h]
+            A = proto_softmax(affinity(Qu[b, h], Kb, scale))
+            dV[t0:t1, h, :] = A.T @ G
+            dA = G @ Vb.T
+            dS = A * (dA - (A * dA).sum(axis=0, keepdims=True))
+            dK[t0:t1, h, :] = scale * (dS.T @ Qu[b, h])
+            dQu[b, h] = scale * (dS @ Kb)
+    return dK, dV, dQu

@@ -299,3 +299,93 @@ ALL_PINS = [
     pin_permutation, pin_ragged_batch, pin_heads_independent, pin_linear_in_v,
     pin_prototype_shift, pin_constant_upstream, pin_fd_fp64,
 ]
+
+
+# ------------------------------------------- per-user queries (Sec. 3.3)
+# Pins of (fwd_uq, bwd_uq) with the signatures of oracle.sa_forward_per_user /
+# oracle.sa_backward_per_user: Q[b, h] per user, dQ[b, h] per user.  They are
+# checked against the shared-query functions, which the pins above fix, and
+# against their own central finite differences.
+
+def _rand_problem_uq(seed, lens, H, P, d):
+    K, V, cu, _, dO = _rand_problem(seed, lens, H, P, d)
+    Qu = _rng(seed + 1000).standard_normal((len(lens), H, P, d))
+    return K, V, cu, Qu, dO
+
+
+def pin_uq_broadcast(fwd_uq, bwd_uq, fwd=None, bwd=None):
+    """The same prototypes for every user: the shared-query results, and the
+    per-user dQ summing to the shared dQ (Sec. 3.1: the prototypes are global)."""
+    from oracle import sa_backward, sa_forward
+
+    lens = [5, 0, 3, 7]
+    K, V, cu, Q, dO = _rand_problem(31, lens, H=2, P=4, d=3)
+    Qu = np.broadcast_to(Q, (len(lens),) + Q.shape).copy()
+    scale = 0.7
+    O_u, lse_u = fwd_uq(K, V, cu, Qu, scale, with_lse=True)
+    O, lse = sa_forward(K, V, cu, Q, scale, with_lse=True)
+    _close(O_u, O, 1e-12, "sketch, broadcast prototypes")
+    _close(lse_u, lse, 1e-12, "lse, broadcast prototypes")
+    dK_u, dV_u, dQ_u = bwd_uq(K, V, cu, Qu, scale, dO)
+    dK, dV, dQ = sa_backward(K, V, cu, Q, scale, dO)
+    _close(dK_u, dK, 1e-12, "dK, broadcast prototypes")
+    _close(dV_u, dV, 1e-12, "dV, broadcast prototypes")
+    _close(dQ_u.sum(axis=0), dQ, 1e-12, "sum over users of per-user dQ")
+    assert np.all(dQ_u[1] == 0), "an empty user has no query gradient"
+
+
+def pin_uq_users_alone(fwd_uq, bwd_uq, fwd=None, bwd=None):
+    """Each user of a ragged batch equals that user alone with the shared-query
+    functions and Q = that user's prototypes."""
+    from oracle import sa_backward, sa_forward
+
+    lens = [6, 2, 0, 9]
+    K, V, cu, Qu, dO = _rand_problem_uq(32, lens, H=2, P=5, d=4)
+    scale = 0.6
+    O_u = fwd_uq(K, V, cu, Qu, scale)
+    dK_u, dV_u, dQ_u = bwd_uq(K, V, cu, Qu, scale, dO)
+    for b in range(len(lens)):
+        t0, t1 = int(cu[b]), int(cu[b + 1])
+        c1 = np.array([0, t1 - t0])
+        O1 = sa_forward(K[t0:t1], V[t0:t1], c1, Qu[b], scale)
+        _close(O_u[b:b + 1], O1, 1e-12, f"sketch of user {b}")
+        dK1, dV1, dQ1 = sa_backward(K[t0:t1], V[t0:t1], c1, Qu[b], scale, dO[b:b + 1])
+        _close(dK_u[t0:t1], dK1, 1e-12, f"dK of user {b}")
+        _close(dV_u[t0:t1], dV1, 1e-12, f"dV of user {b}")
+        _close(dQ_u[b], dQ1, 1e-12, f"dQ of user {b}")
+
+
+def pin_uq_conservation(fwd_uq, bwd_uq=None, fwd=None, bwd=None):
+    """V = 1: every sketch column sums to the user's length (sum_j A[j, i] = 1)."""
+    lens = [4, 0, 11]
+    K, _, cu, Qu, _ = _rand_problem_uq(33, lens, H=3, P=6, d=2)
+    O = fwd_uq(K, np.ones_like(K), cu, Qu, 0.9)
+    for b, L in enumerate(lens):
+        _close(O[b].sum(axis=1), np.full((3, 2), float(L)), 1e-12, f"column sums of user {b}")
+
+
+def pin_uq_fd_fp64(fwd_uq, bwd_uq, fwd=None, bwd=None):
+    """fp64 central differences of the per-user forward, for dQ (per user) and dK."""
+    lens = [7, 5]
+    K, V, cu, Qu, dO = _rand_problem_uq(34, lens, H=2, P=6, d=4)
+    scale = 0.5
+    dK, _, dQ = bwd_uq(K, V, cu, Qu, scale, dO)
+    r = _rng(35)
+
+    def loss(K_, Q_):
+        return float(np.sum(dO * fwd_uq(K_, V, cu, Q_, scale)))
+
+    for name, grad in (("K", dK), ("Q", dQ)):
+        for _ in range(12):
+            idx = tuple(int(r.integers(0, s)) for s in grad.shape)
+            args = {"K": K.copy(), "Q": Qu.copy()}
+            h = 1e-6
+            args[name][idx] += h
+            lp = loss(args["K"], args["Q"])
+            args[name][idx] -= 2 * h
+            lm = loss(args["K"], args["Q"])
+            ref = (lp - lm) / (2 * h)
+            assert abs(grad[idx] - ref) <= 1e-6 * max(1.0, abs(ref)), f"d{name}{idx}"
+
+
+UQ_PINS = [pin_uq_broadcast, pin_uq_users_alone, pin_uq_conservation, pin_uq_fd_fp64]

@@ -3,7 +3,7 @@ import numpy as np
 import pytest
 
 import pins
-from oracle import sa_backward, sa_forward
+from oracle import sa_backward, sa_backward_per_user, sa_forward, sa_forward_per_user
 
 
 @pytest.mark.parametrize("pin", pins.ALL_PINS, ids=lambda p: p.__name__)
@@ -31,3 +31,8 @@ def test_large_scores_do_not_overflow():
     assert np.all(np.isfinite(O)) and np.allclose(O[0, 0].sum() + O[0, 0].sum(), O[0, 0].sum() * 2)
     assert np.allclose(O[0, 0, :, 0].sum(), 2.0)
     assert np.all(np.isfinite(lse))
+
+
+@pytest.mark.parametrize("pin", pins.UQ_PINS, ids=lambda p: p.__name__)
+def test_oracle_per_user_pin(pin):
+    pin(sa_forward_per_user, sa_backward_per_user)

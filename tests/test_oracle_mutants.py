@@ -90,3 +90,39 @@ def test_mutant_is_caught(name):
         except AssertionError:
             caught.append(pin.__name__)
     assert caught, f"no pin catches the planted mistake '{name}'"
+
+
+# ------------------------------------------- per-user queries (Sec. 3.3)
+def _uq_variant(first_user_q=False, dq_summed=False, dq_scale=True):
+    def fwd(K, V, cu, Qu, scale, with_lse=False):
+        Qx = np.broadcast_to(Qu[:1], Qu.shape) if first_user_q else Qu
+        return so.sa_forward_per_user(K, V, cu, np.array(Qx), scale, with_lse=with_lse)
+
+    def bwd(K, V, cu, Qu, scale, dO):
+        Qx = np.array(np.broadcast_to(Qu[:1], Qu.shape)) if first_user_q else Qu
+        dK, dV, dQ = so.sa_backward_per_user(K, V, cu, Qx, scale, dO)
+        if dq_summed:
+            dQ = np.broadcast_to(dQ.sum(axis=0, keepdims=True), dQ.shape).copy()
+        if not dq_scale:
+            dQ = dQ / scale
+        return dK, dV, dQ
+    return fwd, bwd
+
+
+UQ_MUTANTS = {
+    "every user gets user 0's prototypes": _uq_variant(first_user_q=True),
+    "dQ summed over users": _uq_variant(dq_summed=True),
+    "dQ without scale": _uq_variant(dq_scale=False),
+}
+
+
+@pytest.mark.parametrize("name", sorted(UQ_MUTANTS))
+def test_per_user_mutant_is_caught(name):
+    fwd, bwd = UQ_MUTANTS[name]
+    caught = []
+    for pin in pins.UQ_PINS:
+        try:
+            pin(fwd, bwd)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught, f"no pin catches the planted mistake '{name}'"
