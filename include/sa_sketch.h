@@ -93,6 +93,29 @@ sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens,
                         void* dV, float* dQ, void* workspace, size_t ws_bytes,
                         void* stream);
 
+/* Per-user queries, the stacked refinement of Sec. 3.3: from the second SA step
+ * on, the queries are each user's own refined sketch times W_Q^(l), so Q holds
+ * one block of prototypes per user:
+ *     Q : [B, H, P, d]  (type `dt`),    user b, head h reads Q[b, h] instead of Q[h].
+ * Everything else -- arguments, layouts, ownership, `lse`, the workspace size
+ * (sa_workspace_size with the same sizes), errors and determinism -- is as in
+ * sa_sketch_fwd. */
+sa_status sa_sketch_fwd_per_user(const void* K, const void* V, const int32_t* cu_seqlens, int B,
+                                 int64_t N, const void* Q, int H, int P, int d, float scale,
+                                 sa_dtype dt, float* sketch, float* lse, void* workspace,
+                                 size_t ws_bytes, void* stream);
+
+/* Backward with per-user queries (chain rule of Sec. 3.3's steps): as
+ * sa_sketch_bwd, except that Q is [B, H, P, d] and
+ *     dQ : [B, H, P, d] fp32,  dQ[b, h] = scale sum_i dS[:, i] K_b[i, h]
+ * holds only user b's tokens (no sum over the batch); fully overwritten, zero
+ * for a user with L_b = 0. */
+sa_status sa_sketch_bwd_per_user(const void* K, const void* V, const int32_t* cu_seqlens, int B,
+                                 int64_t N, const void* Q, int H, int P, int d, float scale,
+                                 sa_dtype dt, const float* dsketch, const float* lse, void* dK,
+                                 void* dV, float* dQ, void* workspace, size_t ws_bytes,
+                                 void* stream);
+
 /* Allocation-free forward (the paper has no counterpart; this is a library
  * convenience).  For callers that cannot provide a workspace: for example a
  * plugin or custom-operator hook that receives only its input and output

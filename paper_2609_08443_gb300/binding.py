@@ -61,6 +61,10 @@ def load() -> ctypes.CDLL:
     lib.sa_main_kernel_name.restype = ctypes.c_char_p
     lib.sa_select_path.argtypes = [i32]
     lib.sa_select_path.restype = i32
+    lib.sa_sketch_fwd_per_user.argtypes = lib.sa_sketch_fwd.argtypes
+    lib.sa_sketch_fwd_per_user.restype = i32
+    lib.sa_sketch_bwd_per_user.argtypes = lib.sa_sketch_bwd.argtypes
+    lib.sa_sketch_bwd_per_user.restype = i32
     lib.sa_sketch_fwd_noalloc.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp]
     lib.sa_sketch_fwd_noalloc.restype = i32
     lib.sa_noalloc_scratch_bytes.argtypes = []
@@ -98,8 +102,13 @@ def _validate(K, V, cu, Q):
             raise ValueError(f"{name} must be a CUDA tensor")
         if not t.is_contiguous():
             raise ValueError(f"{name} must be contiguous")
-    if K.dim() != 3 or V.shape != K.shape or Q.dim() != 3 or Q.shape[0] != K.shape[1] or Q.shape[2] != K.shape[2]:
-        raise ValueError(f"shapes K{tuple(K.shape)} V{tuple(V.shape)} Q{tuple(Q.shape)}: want K,V [N,H,d], Q [H,P,d]")
+    # Q [H,P,d] (prototypes shared by all users) or [B,H,P,d] (per-user queries, Sec. 3.3)
+    shared_ok = Q.dim() == 3 and Q.shape[0] == K.shape[1] and Q.shape[2] == K.shape[2]
+    per_user_ok = (Q.dim() == 4 and Q.shape[0] == cu.numel() - 1 and Q.shape[1] == K.shape[1]
+                   and Q.shape[3] == K.shape[2])
+    if K.dim() != 3 or V.shape != K.shape or not (shared_ok or per_user_ok):
+        raise ValueError(f"shapes K{tuple(K.shape)} V{tuple(V.shape)} Q{tuple(Q.shape)}: want K,V [N,H,d], "
+                         "Q [H,P,d] or [B,H,P,d]")
     if K.dtype != V.dtype or K.dtype != Q.dtype:
         raise ValueError("K, V and Q must share one dtype")
     if cu.dtype != torch.int32 or cu.dim() != 1 or cu.numel() < 2:
@@ -162,11 +171,13 @@ def sa_sketch_fwd(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q:
                   scale: Optional[float] = None, want_lse: bool = False,
                   out: Optional[torch.Tensor] = None, lse_out: Optional[torch.Tensor] = None,
                   ws: Optional[torch.Tensor] = None):
-    """sketch [B,H,P,d] fp32 (and lse [N,H] fp32 when ``want_lse``)."""
+    """sketch [B,H,P,d] fp32 (and lse [N,H] fp32 when ``want_lse``).  Q is
+    [H,P,d] (C: sa_sketch_fwd) or per user [B,H,P,d] (C: sa_sketch_fwd_per_user)."""
     lib = load()
     _validate(K, V, cu_seqlens, Q)
     N, H, d = K.shape
-    P = Q.shape[1]
+    P = Q.shape[-2]
+    entry = lib.sa_sketch_fwd_per_user if Q.dim() == 4 else lib.sa_sketch_fwd
     B = cu_seqlens.numel() - 1
     dt = _dt(K)
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
@@ -177,20 +188,22 @@ def sa_sketch_fwd(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q:
     if need == 0:
         raise SketchError(2, "sa_workspace_size")
     w = ws if ws is not None else workspace(need, K.device)
-    st = lib.sa_sketch_fwd(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
-                           _ptr(sketch), _ptr(lse), _ptr(w), w.numel(), _stream(K.device))
-    _check(st, "sa_sketch_fwd")
+    st = entry(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
+               _ptr(sketch), _ptr(lse), _ptr(w), w.numel(), _stream(K.device))
+    _check(st, "sa_sketch_fwd_per_user" if Q.dim() == 4 else "sa_sketch_fwd")
     return (sketch, lse) if want_lse or lse_out is not None else sketch
 
 
 def sa_sketch_bwd(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
                   dsketch: torch.Tensor, scale: Optional[float] = None,
                   lse: Optional[torch.Tensor] = None, outs=None, ws: Optional[torch.Tensor] = None):
-    """(dK, dV, dQ): dK, dV like K; dQ [H,P,d] fp32."""
+    """(dK, dV, dQ): dK, dV like K; dQ fp32 shaped like Q ([H,P,d] summed over
+    users, or [B,H,P,d] per user: C sa_sketch_bwd / sa_sketch_bwd_per_user)."""
     lib = load()
     _validate(K, V, cu_seqlens, Q)
     N, H, d = K.shape
-    P = Q.shape[1]
+    P = Q.shape[-2]
+    entry = lib.sa_sketch_bwd_per_user if Q.dim() == 4 else lib.sa_sketch_bwd
     B = cu_seqlens.numel() - 1
     if dsketch.shape != (B, H, P, d) or dsketch.dtype != torch.float32 or not dsketch.is_contiguous():
         raise ValueError("dsketch must be contiguous fp32 [B,H,P,d]")
@@ -200,18 +213,31 @@ def sa_sketch_bwd(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q:
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
     if outs is None:
         dK, dV = torch.empty_like(K), torch.empty_like(V)
-        dQ = torch.empty((H, P, d), dtype=torch.float32, device=K.device)
+        dQ = torch.empty(tuple(Q.shape), dtype=torch.float32, device=K.device)
     else:
         dK, dV, dQ = outs
     need = lib.sa_workspace_size(B, N, H, P, d, dt, 1)
     if need == 0:
         raise SketchError(2, "sa_workspace_size")
     w = ws if ws is not None else workspace(need, K.device)
-    st = lib.sa_sketch_bwd(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
-                           _ptr(dsketch), _ptr(lse), _ptr(dK), _ptr(dV), _ptr(dQ), _ptr(w), w.numel(),
-                           _stream(K.device))
-    _check(st, "sa_sketch_bwd")
+    st = entry(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
+               _ptr(dsketch), _ptr(lse), _ptr(dK), _ptr(dV), _ptr(dQ), _ptr(w), w.numel(), _stream(K.device))
+    _check(st, "sa_sketch_bwd_per_user" if Q.dim() == 4 else "sa_sketch_bwd")
     return dK, dV, dQ
+
+
+def sa_sketch_fwd_per_user(K, V, cu_seqlens, Q, scale=None, **kw):
+    """Forward with per-user queries Q [B,H,P,d] (stacked refinement, Sec. 3.3)."""
+    if Q.dim() != 4:
+        raise ValueError("per-user queries are [B,H,P,d]")
+    return sa_sketch_fwd(K, V, cu_seqlens, Q, scale, **kw)
+
+
+def sa_sketch_bwd_per_user(K, V, cu_seqlens, Q, dsketch, scale=None, **kw):
+    """Backward with per-user queries: dQ [B,H,P,d], each user's own gradient."""
+    if Q.dim() != 4:
+        raise ValueError("per-user queries are [B,H,P,d]")
+    return sa_sketch_bwd(K, V, cu_seqlens, Q, dsketch, scale, **kw)
 
 
 def sa_sketch_fwd_noalloc(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
@@ -224,6 +250,8 @@ def sa_sketch_fwd_noalloc(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Te
     lib = load()
     _validate(K, V, cu_seqlens, Q)
     N, H, d = K.shape
+    if Q.dim() != 3:
+        raise ValueError("sa_sketch_fwd_noalloc takes shared prototypes Q [H,P,d]")
     P = Q.shape[1]
     B = cu_seqlens.numel() - 1
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)

@@ -153,6 +153,8 @@ sa::Args make_args(const void* K, const void* V, const int32_t* cu, int B, int64
   a.partial = reinterpret_cast<float*>(base + L.partial);
   a.dq_partial = reinterpret_cast<float*>(base + L.dq_partial);
   a.lse_scratch = reinterpret_cast<float*>(base + L.lse);
+  a.uq = 0;
+  a.dq_user = nullptr;
   return a;
 }
 
@@ -232,14 +234,20 @@ size_t sa_workspace_size(int B, int64_t N, int H, int P, int d, sa_dtype dt, int
   return make_plan(B, N, H, P, d, dt, bwd != 0).lay.total;
 }
 
-sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
-                        const void* Q, int H, int P, int d, float scale, sa_dtype dt, float* sketch,
-                        float* lse, void* workspace, size_t ws_bytes, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Forward of both entry points; uq = 1: Q holds one [H, P, d] block per user.
+sa_status fwd_impl(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N, const void* Q, int H,
+                   int P, int d, float scale, sa_dtype dt, float* sketch, float* lse, void* workspace,
+                   size_t ws_bytes, void* stream, int uq) {
   if (!sketch) return SA_ERR_INVALID_ARG;
   Plan plan;
   SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, false, &plan));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, plan.lay);
+  a.uq = uq;
   char* base = static_cast<char*>(workspace);
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, plan.T_fwd, st); }));
   if (plan.fwd_path == Path::TcFwd) {
@@ -258,15 +266,24 @@ sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens,
   return SA_OK;
 }
 
-sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
-                        const void* Q, int H, int P, int d, float scale, sa_dtype dt, const float* dsketch,
-                        const float* lse, void* dK, void* dV, float* dQ, void* workspace, size_t ws_bytes,
-                        void* stream) {
+// Backward of both entry points; uq = 1: Q and dQ hold one [H, P, d] block per
+// user, whose pieces from different workers are summed like the sketch's.
+sa_status bwd_impl(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N, const void* Q, int H,
+                   int P, int d, float scale, sa_dtype dt, const float* dsketch, const float* lse, void* dK,
+                   void* dV, float* dQ, void* workspace, size_t ws_bytes, void* stream, int uq) {
   if (!dsketch || !dQ || (N > 0 && (!dK || !dV))) return SA_ERR_INVALID_ARG;
   Plan plan;
   SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, true, &plan));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, plan.lay);
+  a.uq = uq;
+  a.dq_user = uq ? dQ : nullptr;
+  // dQ from the per-worker pieces: summed over workers per head (shared
+  // queries) or, per user, only for segments cut across workers
+  auto finalize_dq = [&](int W) -> sa_status {
+    if (uq) return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_sketch(a, W, dQ, st); });
+    return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, W, dQ, st); });
+  };
   char* base = static_cast<char*>(workspace);
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, plan.T_bwd, st); }));
   const float* l = lse;
@@ -288,8 +305,7 @@ sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens,
     SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
                   [&] { return sa::launch_tc_bwd_tok(a, plan.W_bwd, dsketch, gbf, l, Dco, dK, dV, st); }));
     SA_TRY(launch(SA_KERNEL_BWD_DQ, st, [&] { return sa::launch_tc_bwd_dq(a, Wq, dsketch, l, Dco, st); }));
-    SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, Wq, dQ, st); }));
-    return SA_OK;
+    return finalize_dq(Wq);
   }
   if (plan.bwd_path == Path::TcBwd) {
     SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
@@ -300,8 +316,39 @@ sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens,
                   [&] { return sa::launch_simt_bwd_tokens(a, dsketch, l, dK, dV, Dco, st); }));
     SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_simt_bwd_dq(a, plan.W_bwd, dsketch, l, Dco, st); }));
   }
-  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, plan.W_bwd, dQ, st); }));
-  return SA_OK;
+  return finalize_dq(plan.W_bwd);
+}
+
+}  // namespace
+
+extern "C" {
+
+sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                        const void* Q, int H, int P, int d, float scale, sa_dtype dt, float* sketch,
+                        float* lse, void* workspace, size_t ws_bytes, void* stream) {
+  return fwd_impl(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, sketch, lse, workspace, ws_bytes, stream, 0);
+}
+
+sa_status sa_sketch_bwd(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                        const void* Q, int H, int P, int d, float scale, sa_dtype dt, const float* dsketch,
+                        const float* lse, void* dK, void* dV, float* dQ, void* workspace, size_t ws_bytes,
+                        void* stream) {
+  return bwd_impl(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, dsketch, lse, dK, dV, dQ, workspace, ws_bytes,
+                  stream, 0);
+}
+
+sa_status sa_sketch_fwd_per_user(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                                 const void* Q, int H, int P, int d, float scale, sa_dtype dt, float* sketch,
+                                 float* lse, void* workspace, size_t ws_bytes, void* stream) {
+  return fwd_impl(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, sketch, lse, workspace, ws_bytes, stream, 1);
+}
+
+sa_status sa_sketch_bwd_per_user(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                                 const void* Q, int H, int P, int d, float scale, sa_dtype dt, const float* dsketch,
+                                 const float* lse, void* dK, void* dV, float* dQ, void* workspace,
+                                 size_t ws_bytes, void* stream) {
+  return bwd_impl(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, dsketch, lse, dK, dV, dQ, workspace, ws_bytes,
+                  stream, 1);
 }
 
 sa_status sa_get_device_error(const void* workspace, void* stream) {

@@ -20,7 +20,12 @@ struct Args {
   float* partial;      // [W][2][P][d]
   float* dq_partial;   // [W][H][P][d]
   float* lse_scratch;  // [N][H] workspace copy of lse when the caller passes none
+  int uq;              // 1: per-user queries Q[B][H][P][d] and dQ[B][H][P][d] (stacked refinement)
+  float* dq_user;      // per-user queries: the caller's dQ[B][H][P][d] (whole segments go there)
 };
+
+// Row of Q ([H or B*H][P][d]) that user b, head h reads.
+SA_HD int q_row(const Args& a, int b, int h) { return a.uq ? b * a.H + h : h; }
 
 // planner / finalize (sa_simt.cu)
 cudaError_t launch_plan(const Args& a, int T, cudaStream_t st);

@@ -175,12 +175,25 @@ __device__ __forceinline__ void stage_rows_f32(float* dst, const float* src, int
   }
 }
 
+// User of token t: the largest b with cu[b] <= t (empty users before it share
+// its offset, so the largest such b is the user that holds t).
+__device__ __forceinline__ int user_of_token(const int32_t* cu, int B, int64_t t) {
+  int lo = 0, hi = B - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (int64_t(cu[mid]) <= t) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
 // ----------------------------------------------------------- lse (forward)
-// One warp per (token, head): lse = log sum_j exp(scale * q_j . k).
+// One warp per (token, head): lse = log sum_j exp(scale * q_j . k), with the
+// token's user's prototypes when the queries are per user.
 template <typename T>
 __global__ void __launch_bounds__(256) simt_lse_kernel(const T* __restrict__ K, const T* __restrict__ Q,
                                                        int64_t N, int H, int P, int d, float scale,
-                                                       float* __restrict__ lse, const void* ws) {
+                                                       float* __restrict__ lse, const void* ws,
+                                                       const int32_t* __restrict__ cu, int B, int uq) {
   __shared__ float ks[8][kMaxD];
   if (ws_failed(ws)) return;
   const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
@@ -193,8 +206,9 @@ __global__ void __launch_bounds__(256) simt_lse_kernel(const T* __restrict__ K, 
   __syncwarp();
   constexpr int VN = Vec<T>::n;
   float m = -INFINITY, z = 0.f;
+  const int qr = uq ? user_of_token(cu, B, t) * H + h : h;
   for (int j = lane; j < P; j += 32) {
-    const T* q = Q + (int64_t(h) * P + j) * d;
+    const T* q = Q + (int64_t(qr) * P + j) * d;
     float s = 0.f;
     for (int c = 0; c < d; c += VN) {
       float v[VN];
@@ -250,13 +264,14 @@ __global__ void __launch_bounds__(SNT) simt_fwd_agg_kernel(Args a, const float* 
   float acc[kMaxD / 4];
 #pragma unroll
   for (int m = 0; m < kMaxD / 4; ++m) acc[m] = 0.f;
-  int cur_h = -1;
+  int cur_q = -1;
   for (int64_t t = tb; t < te; ++t) {
     const TileRef r = locate_tile(t, tph, a.prefix, a.cu, a.B, ST);
     __syncthreads();
-    if (r.h != cur_h) {
-      stage_rows(Qs, Q + (int64_t(r.h) * P + p0) * d, d, np, SPB, d);
-      cur_h = r.h;
+    const int qr = q_row(a, r.b, r.h);
+    if (qr != cur_q) {
+      stage_rows(Qs, Q + (int64_t(qr) * P + p0) * d, d, np, SPB, d);
+      cur_q = qr;
     }
     stage_rows(Ks, K + (r.tok0 * H + r.h) * int64_t(d), int64_t(H) * d, r.n, ST, d);
     stage_rows(Vs, V + (r.tok0 * H + r.h) * int64_t(d), int64_t(H) * d, r.n, ST, d);
@@ -342,7 +357,7 @@ __global__ void __launch_bounds__(SNT) simt_bwd_tokens_kernel(Args a, const floa
   for (int pc = 0; pc < P; pc += SPB) {
     const int np = min(SPB, P - pc);
     __syncthreads();
-    stage_rows(Qs, Q + (int64_t(r.h) * P + pc) * d, d, np, SPB, d);
+    stage_rows(Qs, Q + (int64_t(q_row(a, r.b, r.h)) * P + pc) * d, d, np, SPB, d);
     stage_rows_f32(Gs, G + int64_t(pc) * d, np, SPB, d);
     __syncthreads();
     {
@@ -395,7 +410,7 @@ __global__ void __launch_bounds__(SNT) simt_bwd_tokens_kernel(Args a, const floa
   for (int pc = 0; pc < P; pc += SPB) {
     const int np = min(SPB, P - pc);
     __syncthreads();
-    stage_rows(Qs, Q + (int64_t(r.h) * P + pc) * d, d, np, SPB, d);
+    stage_rows(Qs, Q + (int64_t(q_row(a, r.b, r.h)) * P + pc) * d, d, np, SPB, d);
     stage_rows_f32(Gs, G + int64_t(pc) * d, np, SPB, d);
     __syncthreads();
     {
@@ -467,11 +482,13 @@ __global__ void __launch_bounds__(SNT) simt_bwd_dq_kernel(Args a, const float* _
   float acc[kMaxD / 4];
 #pragma unroll
   for (int m = 0; m < kMaxD / 4; ++m) acc[m] = 0.f;
-  int cur_h = -1, cur_b = -1;
+  int cur_h = -1, cur_b = -1, cur_q = -1;
   for (int64_t t = tb; t < te; ++t) {
     const TileRef r = locate_tile(t, tph, a.prefix, a.cu, a.B, ST);
     __syncthreads();
-    if (r.h != cur_h) stage_rows(Qs, Q + (int64_t(r.h) * P + p0) * d, d, np, SPB, d);
+    const int qr = q_row(a, r.b, r.h);
+    if (qr != cur_q) stage_rows(Qs, Q + (int64_t(qr) * P + p0) * d, d, np, SPB, d);
+    cur_q = qr;
     if (r.h != cur_h || r.b != cur_b)
       stage_rows_f32(Gs, dsk + ((int64_t(r.b) * H + r.h) * P + p0) * d, np, SPB, d);
     cur_h = r.h;
@@ -511,8 +528,19 @@ __global__ void __launch_bounds__(SNT) simt_bwd_dq_kernel(Args a, const float* _
         if (c < d) acc[m] = fmaf(ds, Ks[i * dp + c], acc[m]);
       }
     }
-    if (t + 1 == te || (t + 1) / tph != t / tph) {  // head ends: flush
-      float* dst = a.dq_partial + ((int64_t(w) * H + r.h) * P + p0 + p) * d;
+    // flush where the row of Q changes: at a head's end (shared queries: the
+    // worker's partial of head h) or at a user segment's end (per-user queries:
+    // dQ[b, h] when this worker holds the whole segment, else its partial slot)
+    const bool flush = a.uq ? (t + 1 == te || t + 1 == r.seg1) : (t + 1 == te || (t + 1) / tph != t / tph);
+    if (flush) {
+      float* dst;
+      if (!a.uq) {
+        dst = a.dq_partial + ((int64_t(w) * H + r.h) * P + p0 + p) * d;
+      } else if (r.seg0 >= tb && r.seg1 <= te) {
+        dst = a.dq_user + ((int64_t(r.b) * H + r.h) * P + p0 + p) * d;
+      } else {
+        dst = a.partial + ((int64_t(w) * 2 + partial_slot(total, W, w, r.seg0)) * P + p0 + p) * d;
+      }
 #pragma unroll
       for (int m = 0; m < kMaxD / 4; ++m) {
         const int c = cq + 4 * m;
@@ -557,11 +585,11 @@ cudaError_t launch_simt_lse(const Args& a, float* lse, cudaStream_t st) {
   if (a.dt == SA_BF16)
     simt_lse_kernel<__nv_bfloat16><<<unsigned(blocks), 256, 0, st>>>(
         static_cast<const __nv_bfloat16*>(a.K), static_cast<const __nv_bfloat16*>(a.Q), a.N, a.H, a.P, a.d,
-        a.scale, lse, a.ws);
+        a.scale, lse, a.ws, a.cu, a.B, a.uq);
   else
     simt_lse_kernel<float><<<unsigned(blocks), 256, 0, st>>>(static_cast<const float*>(a.K),
                                                              static_cast<const float*>(a.Q), a.N, a.H, a.P,
-                                                             a.d, a.scale, lse, a.ws);
+                                                             a.d, a.scale, lse, a.ws, a.cu, a.B, a.uq);
   return cudaGetLastError();
 }
 

@@ -162,13 +162,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t e = 0;
       bool ok = true;
       for (int li = 0; li < ntiles && ok; ++li) {
-        if (it.h != prev_h) {
+        if (it.qk != prev_h) {  // a new head (or, with per-user queries, a new user)
           if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0x401);
           if (!ok) break;
           mbar_arrive_expect_tx(q_full, C::Q_BYTES);
 #pragma unroll
-          for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.h);
-          prev_h = it.h;
+          for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.qk);
+          prev_h = it.qk;
           ++hc;
         }
 #pragma unroll
@@ -220,7 +220,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         issue_S(0, sdcol(0));
         umma_commit(s_full);
         // slice mode: Q is read only by S, so it may be replaced after the last S of a head
-        if (MODE == kSlice && (ntiles == 1 || nxt.h != cur.h)) umma_commit(q_empty);
+        if (MODE == kSlice && (ntiles == 1 || nxt.qk != cur.qk)) umma_commit(q_empty);
       }
       bool first_of_hp = true;
       for (int li = 0; li < ntiles && ok; ++li) {
@@ -259,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         if (cur.seg_last) umma_commit(g_empty);
         const bool more = li + 1 < ntiles;
-        const bool newhead = more && nxt.h != cur.h;
+        const bool newhead = more && nxt.qk != cur.qk;
         // ---- S(i+1) before dK/dQ(i) when its buffer and Q allow it
         const bool early = more && (C::NSD == 2 || !newhead);
         if (early) {
@@ -277,7 +277,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
           issue_S((eK + 2) % C::NSLOT, sdcol(li + 1));
           umma_commit(s_full);
-          if (MODE == kSlice && (li + 2 >= ntiles || nx2.h != nxt.h)) umma_commit(q_empty);
+          if (MODE == kSlice && (li + 2 >= ntiles || nx2.qk != nxt.qk)) umma_commit(q_empty);
         }
         // ---- dK(i) = dS Q, dQ += dS^T K
         wt(ds_full, li & 1, 0x50B);
@@ -378,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) mbar_arrive(dk_empty);
         }
         if (last_of_hp) {
-          float* dst = a.dq_partial + ((int64_t(wk) * a.H + pw.h) * a.P + p0) * D;
+          float* dst = dq_block_dst(a, wk, W, total, pw, p0, D);
           store_sketch_scaled<D, PS, C::DQ_COL>(tmem, lane_off, sw, q, lane, dst, a.scale);
           tc_fence_before();
           __syncwarp();
@@ -431,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = wwait(ab_empty, (li - 1) & 1, 0x702);
           if (!ok) break;
           tc_fence_after();
-          finish_prev(prev, prev.h != cur.h);
+          finish_prev(prev, prev.qk != cur.qk);
           prev.next();
         }
         // ---- A -> shared memory [PS/64][128 tokens][64], 128-byte swizzle
@@ -548,7 +548,7 @@ static cudaError_t launch_bwd_t(const Args& a, int W, const float* dsk, const fl
   using C = BCfg<D, PS, MODE>;
   CUtensorMap tk, tv, tq;
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
-      !make_q_map(&tq, a.Q, a.H, a.P, D, PS))
+      !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, PS))
     return cudaErrorInvalidValue;
   auto fn = &tc_bwd_kernel<D, PS, MODE>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -733,7 +733,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int li = 0; li < ntiles && ok; ++li) {
         for (int c = 0; c < C::NCH && ok; ++c) {
           const int pr = tok_qg_pair(li, c);
-          load(2 * pr + 1, &tmQ, c * C::NC, it.h);
+          load(2 * pr + 1, &tmQ, c * C::NC, it.qk);
           load(2 * pr, &tmG, c * C::NC, int(it.b) * a.H + it.h);
           if (c == 0 && li > 0) load(1, &tmV, it.h, int(it.tok0));
           if (c == C::NCH - 1 && li + 1 < ntiles) load(0, &tmK, nx.h, int(nx.tok0));
@@ -1060,7 +1060,7 @@ static cudaError_t launch_tok_t(const Args& a, int W, const __nv_bfloat16* gbf, 
   using C = TokCfg<D, P>;
   CUtensorMap tk, tv, tq, tg, tdk, tdv;
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
-      !make_q_map(&tq, a.Q, a.H, a.P, D, C::NC) || !make_q_map(&tg, gbf, a.B * a.H, a.P, D, C::NC) ||
+      !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, C::NC) || !make_q_map(&tg, gbf, a.B * a.H, a.P, D, C::NC) ||
       !make_kv_map(&tdk, dK, a.N, a.H, D) || !make_kv_map(&tdv, dV, a.N, a.H, D))
     return cudaErrorInvalidValue;
   auto fn = &tc_bwd_tok_kernel<D, P>;
@@ -1213,20 +1213,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       int hc = 0, prev_h = -1, loaded = 0;
       bool ok = true;
       for (int li = 0; li < ntiles && ok; ++li) {
-        const bool new_head = it.h != prev_h;
+        // "head" below = the run of tiles reading one row of Q: a head, or with
+        // per-user queries one (user, head) segment
+        const bool new_head = it.qk != prev_h;
         if (new_head) {
           if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0xC01);
           if (!ok) break;
           mbar_arrive_expect_tx(q_full, C::QB);
 #pragma unroll
-          for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.h);
-          prev_h = it.h;
+          for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.qk);
+          prev_h = it.qk;
           ++hc;
         }
         int64_t t0n;
-        int nn, hn;
-        it.peek_next(t0n, nn, hn);
-        const uint32_t fl = (new_head ? kNewHead : 0u) | ((li + 1 >= ntiles || hn != it.h) ? kHeadLast : 0u) |
+        int nn, hn, qkn;
+        it.peek_next(t0n, nn, hn, qkn);
+        const uint32_t fl = (new_head ? kNewHead : 0u) | ((li + 1 >= ntiles || qkn != it.qk) ? kHeadLast : 0u) |
                             (it.seg_first ? kSegFirst : 0u) | (it.seg_last ? kSegLast : 0u);
 #pragma unroll
         for (int kv = 0; kv < 2; ++kv) {
@@ -1425,16 +1427,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive(ds_full);
           mbar_arrive(col_empty0 + 8 * buf);
         }
-        // dQ partial of this worker and head at the end of its head piece
+        // dQ partial of this worker and head (or user segment) at the end of its piece
         const bool more = li + 1 < ntiles;
         int64_t t0n;
-        int nn, hn;
-        cur.peek_next(t0n, nn, hn);
-        if (!more || hn != cur.h) {
+        int nn, hn, qkn;
+        cur.peek_next(t0n, nn, hn, qkn);
+        if (!more || qkn != cur.qk) {
           ok = wwait(ds_empty0 + 8 * buf, (li >> 1) & 1, 0xF05);
           if (!ok) break;
           tc_fence_after();
-          float* dst = a.dq_partial + ((int64_t(wk) * a.H + cur.h) * a.P + p0) * D;
+          float* dst = dq_block_dst(a, wk, W, total, cur, p0, D);
           store_sketch_scaled<D, PS, C::DQ_COL>(tmem, lane_off, sw, q, lane, dst, a.scale);
           tc_fence_before();
           __syncwarp();
@@ -1459,7 +1461,7 @@ static cudaError_t launch_dq_t(const Args& a, int W, const float* dsk, const flo
   using C = QCfg<D, PS>;
   CUtensorMap tk, tv, tq;
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
-      !make_q_map(&tq, a.Q, a.H, a.P, D, PS))
+      !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, PS))
     return cudaErrorInvalidValue;
   auto fn = &tc_bwd_dq_kernel<D, PS>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);

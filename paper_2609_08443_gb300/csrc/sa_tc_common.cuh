@@ -24,16 +24,17 @@ __host__ __device__ constexpr int tmem_cols_for(int c) {
 struct TileWalker {
   const int64_t* prefix;
   const int32_t* cu;
-  int B, Tt;
+  int B, Tt, H, uq;
   int64_t tph, t, tb, te;
   int h, b;
+  int qk;  // row of Q this tile reads: h (shared queries) or b*H + h (per user)
   int64_t k, nk, tok0, seg0, seg1;
   int64_t cub, Lb;  // cu[b] and L_b of the current user, read once per segment
   int n;
   bool seg_first, seg_last;
 
   __device__ TileWalker(const Args& a, int64_t tb_, int64_t te_, int T_)
-      : prefix(a.prefix), cu(a.cu), B(a.B), Tt(T_), t(tb_), tb(tb_), te(te_) {
+      : prefix(a.prefix), cu(a.cu), B(a.B), Tt(T_), H(a.H), uq(a.uq), t(tb_), tb(tb_), te(te_) {
     tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
     if (t < te) relocate();
   }
@@ -41,6 +42,7 @@ struct TileWalker {
     const TileRef r = locate_tile(t, tph, prefix, cu, B, Tt);
     h = r.h;
     b = r.b;
+    qk = uq ? b * H + h : h;
     seg0 = r.seg0;
     seg1 = r.seg1;
     nk = seg1 - seg0;
@@ -58,10 +60,16 @@ struct TileWalker {
   }
   // First token, size and head of the tile after this one (n = 0 past the range).
   __device__ void peek_next(int64_t& tok0_n, int& n_n, int& h_n) const {
+    int qk_n;
+    peek_next(tok0_n, n_n, h_n, qk_n);
+  }
+  // ... and the row of Q it reads (qk_n = qk past the range)
+  __device__ void peek_next(int64_t& tok0_n, int& n_n, int& h_n, int& qk_n) const {
     if (t + 1 >= te) {
       tok0_n = 0;
       n_n = 0;
       h_n = h;
+      qk_n = qk;
       return;
     }
     if (k + 1 < nk) {
@@ -69,11 +77,13 @@ struct TileWalker {
       const int64_t left = Lb - (k + 1) * Tt;
       n_n = int(left < Tt ? left : Tt);
       h_n = h;
+      qk_n = qk;
     } else {
       const TileRef r = locate_tile(t + 1, tph, prefix, cu, B, Tt);
       tok0_n = r.tok0;
       n_n = r.n;
       h_n = r.h;
+      qk_n = uq ? r.b * H + r.h : r.h;
     }
   }
   __device__ void next() {
@@ -87,6 +97,18 @@ struct TileWalker {
     }
   }
 };
+
+// Where a worker's dQ block of prototypes [p0, p0 + PS) for the tiles ending
+// at walker position w goes.  Shared queries: the worker's partial of head h
+// ([W][H][P][d], summed over workers afterwards).  Per-user queries: dQ[b, h]
+// itself when the worker holds the whole (user, head) segment, else the
+// worker's partial slot of that segment ([W][2][P][d], summed like the sketch).
+__device__ __forceinline__ float* dq_block_dst(const Args& a, int wk, int W, int64_t total, const TileWalker& w,
+                                               int p0, int D) {
+  if (!a.uq) return a.dq_partial + ((int64_t(wk) * a.H + w.h) * a.P + p0) * D;
+  if (w.seg0 >= w.tb && w.seg1 <= w.te) return a.dq_user + ((int64_t(w.b) * a.H + w.h) * a.P + p0) * D;
+  return a.partial + ((int64_t(wk) * 2 + partial_slot(total, W, wk, w.seg0)) * a.P + p0) * D;
+}
 
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
   if (ptx::mbar_try_wait(bar, parity)) return true;

@@ -169,13 +169,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           pf.next();
         }
         if (li < ntiles) {
-          if (it.h != prev_h) {
+          if (it.qk != prev_h) {  // a new head (or, with per-user queries, a new user)
             if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0x101);
             if (!ok) break;
             mbar_arrive_expect_tx(q_full, C::Q_BYTES);
 #pragma unroll
-            for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.h);
-            prev_h = it.h;
+            for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(sQ + dh * PS * 128, &tmQ, q_full, 64 * dh, p0, it.qk);
+            prev_h = it.qk;
             ++hc;
           }
           const int s = int(e % C::NSLOT);
@@ -230,13 +230,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_S(0);
           umma_commit(s_full);
           umma_commit(ring_empty(0));
-          if (ntiles == 1 || nxt.h != cur.h) umma_commit(q_empty);
+          if (ntiles == 1 || nxt.qk != cur.qk) umma_commit(q_empty);
           e = 1;
         }
       }
       for (int li = 0; li < ntiles && ok; ++li) {
         if (li + 1 < ntiles) {
-          if (nxt.h != cur.h) {
+          if (nxt.qk != cur.qk) {
             ++hc;
             ok = mbar_wait(q_full, hc & 1, abort_flag, a.ws, 0x203);
             if (!ok) break;
@@ -251,10 +251,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_commit(s_full);
           umma_commit(ring_empty(s));
           ++e;
-          // last S of this head: Q may be replaced once it completes
-          const int h_now = nxt.h;
+          // last S of these prototypes: Q may be replaced once it completes
+          const int q_now = nxt.qk;
           nxt.next();
-          if (li + 2 >= ntiles || nxt.h != h_now) umma_commit(q_empty);
+          if (li + 2 >= ntiles || nxt.qk != q_now) umma_commit(q_empty);
         }
         // aggregation of tile li
         ok = mbar_wait(w_full, li & 1, abort_flag, a.ws, 0x206);
@@ -533,7 +533,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t e = 0;
       bool ok = true;
       for (int li = 0; li < ntiles && ok; ++li) {
-        if (it.h != prev_h) {
+        if (it.qk != prev_h) {
           if (hc > 0) ok = mbar_wait(q_empty, (hc - 1) & 1, abort_flag, a.ws, 0x111);
           if (!ok) break;
           mbar_arrive_expect_tx(q_full, C::Q_BYTES);
@@ -541,8 +541,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < NCH; ++c)
 #pragma unroll
             for (int dh = 0; dh < D / 64; ++dh)
-              tma_load_3d(sQ + dh * C::P * 128 + c * NC * 128, &tmQ, q_full, 64 * dh, c * NC, it.h);
-          prev_h = it.h;
+              tma_load_3d(sQ + dh * C::P * 128 + c * NC * 128, &tmQ, q_full, 64 * dh, c * NC, it.qk);
+          prev_h = it.qk;
           ++hc;
         }
         const int s = int(e % C::NSLOT);
@@ -566,7 +566,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       uint32_t g = 0;  // (tile, chunk) counter
       for (int li = 0; li < ntiles && ok; ++li) {
-        const int h_now = cur.h;
+        const int h_now = cur.qk;
         if (h_now != prev_h) {
           prev_h = h_now;
           ok = mbar_wait(q_full, hc & 1, abort_flag, a.ws, 0x211);
@@ -593,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         umma_commit(ring_empty(s));
         cur.next();
-        if (li + 1 >= ntiles || cur.h != h_now) umma_commit(q_empty);
+        if (li + 1 >= ntiles || cur.qk != h_now) umma_commit(q_empty);
       }
       umma_commit(drain);
       mbar_wait_bounded(drain, 0, 200000000ull);
@@ -668,7 +668,7 @@ static cudaError_t launch_fwd_t(const Args& a, int W, float* sketch, float* lse_
   using C = Cfg<D, PS, MODE>;
   CUtensorMap tk, tv, tq;
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
-      !make_q_map(&tq, a.Q, a.H, a.P, D, PS))
+      !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, PS))
     return cudaErrorInvalidValue;
   auto fn = &tc_fwd_kernel<D, PS, MODE>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -698,7 +698,8 @@ template <int D, int NC, int NCH>
 static cudaError_t launch_lse_t(const Args& a, int W, float* lse_out, cudaStream_t st) {
   using C = LseCfg<D, NC, NCH>;
   CUtensorMap tk, tq;
-  if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_q_map(&tq, a.Q, a.H, a.P, D, NC)) return cudaErrorInvalidValue;
+  if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, NC))
+    return cudaErrorInvalidValue;
   auto fn = &tc_lse_kernel<D, NC, NCH>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;

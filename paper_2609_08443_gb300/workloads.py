@@ -153,7 +153,8 @@ def _user_rows(spec: Spec, user_id: int, L: int, which: int) -> np.ndarray:
     return _stream(spec, 11, which, user_id).standard_normal((L, spec.H, spec.d), dtype=np.float32)
 
 
-def make_host(spec: Spec, users: Optional[Sequence[int]] = None) -> Dict[str, np.ndarray]:
+def make_host(spec: Spec, users: Optional[Sequence[int]] = None,
+              per_user_q: bool = False) -> Dict[str, np.ndarray]:
     """Draw the workload on the host.
 
     Returns fp32 arrays for F32 specs and uint16 bf16 bit patterns for BF16
@@ -161,6 +162,9 @@ def make_host(spec: Spec, users: Optional[Sequence[int]] = None) -> Dict[str, np
     "lengths" and "users" (the original user indices kept).
     ``users`` restricts the batch to a subset of the spec's users; each user's
     rows are identical to the ones it has in the full batch.
+    ``per_user_q`` replaces Q by per-user prototypes [B, H, P, d] (the queries of
+    the stacked refinement steps), drawn from one stream per user with the same
+    standard deviation.
     """
     lens_all = lengths(spec)
     users = list(range(spec.B)) if users is None else [int(u) for u in users]
@@ -170,8 +174,12 @@ def make_host(spec: Spec, users: Optional[Sequence[int]] = None) -> Dict[str, np
     empty = np.zeros((0, spec.H, spec.d), dtype=np.float32)
     K = np.concatenate(parts_k) if parts_k else empty
     V = np.concatenate(parts_v) if parts_v else empty
-    Q = _stream(spec, 13).standard_normal((spec.H, spec.P, spec.d), dtype=np.float32)
-    Q = (Q * np.float32(spec.q_std)).astype(np.float32)
+    if per_user_q:
+        Q = np.stack([_stream(spec, 19, u).standard_normal((spec.H, spec.P, spec.d), dtype=np.float32)
+                      for u in users]) if users else np.zeros((0, spec.H, spec.P, spec.d), np.float32)
+    else:
+        Q = _stream(spec, 13).standard_normal((spec.H, spec.P, spec.d), dtype=np.float32)
+    Q = np.ascontiguousarray((Q * np.float32(spec.q_std)).astype(np.float32))
     dS = np.stack([_stream(spec, 17, u).standard_normal((spec.H, spec.P, spec.d), dtype=np.float32)
                    for u in users]) if users else np.zeros((0, spec.H, spec.P, spec.d), np.float32)
     out = {"cu_seqlens": cu_seqlens(lens), "lengths": lens, "users": np.asarray(users),

@@ -4,7 +4,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from oracle import sa_backward, sa_forward
+from oracle import sa_backward, sa_backward_per_user, sa_forward, sa_forward_per_user
 from paper_2609_08443_gb300 import workloads as wl
 
 TOL = {wl.F32: 1e-4, wl.BF16: 2e-2}  # max|gpu - oracle| <= TOL * max|oracle|
@@ -34,10 +34,12 @@ def oracle_outputs(spec, host, bwd=True):
     V = wl.host_as_f64(spec, host["V"])
     Q = wl.host_as_f64(spec, host["Q"])
     cu = host["cu_seqlens"]
-    O, lse = sa_forward(K, V, cu, Q, spec.scale, with_lse=True)
+    per_user = Q.ndim == 4  # per-user queries of the stacked refinement (Sec. 3.3)
+    fwd, bwd_fn = (sa_forward_per_user, sa_backward_per_user) if per_user else (sa_forward, sa_backward)
+    O, lse = fwd(K, V, cu, Q, spec.scale, with_lse=True)
     out = {"sketch": O, "lse": lse}
     if bwd:
-        dK, dV, dQ = sa_backward(K, V, cu, Q, spec.scale, host["dsketch"].astype(np.float64))
+        dK, dV, dQ = bwd_fn(K, V, cu, Q, spec.scale, host["dsketch"].astype(np.float64))
         out.update(dK=dK, dV=dV, dQ=dQ)
     return out
 
@@ -57,10 +59,10 @@ def gpu_outputs(spec, t, bwd=True, pass_lse=True):
     return {k: wl.torch_as_f64(v) for k, v in out.items()}
 
 
-def check_spec(spec, bwd=True, pass_lse=True, users=None):
+def check_spec(spec, bwd=True, pass_lse=True, users=None, per_user_q=False):
     import torch
 
-    host = wl.make_host(spec, users=users)
+    host = wl.make_host(spec, users=users, per_user_q=per_user_q)
     t = wl.host_to_torch(spec, host, torch.device("cuda"))
     got = gpu_outputs(spec, t, bwd=bwd, pass_lse=pass_lse)
     ref = oracle_outputs(spec, host, bwd=bwd)
