@@ -68,7 +68,7 @@ typedef enum { SA_F32 = 0, SA_BF16 = 1 } sa_dtype;
 /* Bytes of scratch the caller must pass as `workspace` (device memory, 256-byte
  * aligned) for a call with these sizes on the current device; `bwd` != 0 sizes
  * it for sa_sketch_bwd, which needs more.  Returns 0 for invalid sizes.
- * Supported: 1 <= P <= 1024, 1 <= d <= 128 (d a multiple of 8 for bf16, of 4 for
+ * Supported: 1 <= P <= 2048, 1 <= d <= 128 (d a multiple of 8 for bf16, of 4 for
  * f32), 1 <= H <= 64, B >= 1, 0 <= N < 2^31. */
 size_t sa_workspace_size(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd);
 

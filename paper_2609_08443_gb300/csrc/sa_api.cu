@@ -153,6 +153,7 @@ sa::Args make_args(const void* K, const void* V, const int32_t* cu, int B, int64
   a.partial = reinterpret_cast<float*>(base + L.partial);
   a.dq_partial = reinterpret_cast<float*>(base + L.dq_partial);
   a.lse_scratch = reinterpret_cast<float*>(base + L.lse);
+  a.lse_part = reinterpret_cast<float2*>(base + L.lse_part);
   a.uq = 0;
   a.dq_user = nullptr;
   return a;

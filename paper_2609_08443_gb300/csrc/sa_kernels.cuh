@@ -20,6 +20,7 @@ struct Args {
   float* partial;      // [W][2][P][d]
   float* dq_partial;   // [W][H][P][d]
   float* lse_scratch;  // [N][H] workspace copy of lse when the caller passes none
+  float2* lse_part;    // [N][H][slices] per-slice (max, sum) of the lse pass when P >= 1024
   int uq;              // 1: per-user queries Q[B][H][P][d] and dQ[B][H][P][d] (stacked refinement)
   float* dq_user;      // per-user queries: the caller's dQ[B][H][P][d] (whole segments go there)
 };

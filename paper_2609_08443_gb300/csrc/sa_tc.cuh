@@ -6,6 +6,7 @@ namespace sa {
 
 bool tc_fwd_supported(int P, int d, sa_dtype dt);
 bool tc_fwd_needs_lse_pass_d(int P, int d);  // lse pass, then 256-prototype slices
+int tc_lse_slice(int P, int d);              // prototypes per slice of the lse pass
 bool tc_path_enabled();
 bool tc_fwd_sliced_selected();  // sa_select_path(2)
 bool tc_bwd_supported(int P, int d, sa_dtype dt);

@@ -565,11 +565,14 @@ static cudaError_t launch_bwd_t(const Args& a, int W, const float* dsk, const fl
 // accumulators fit (d = 64 with P <= 256, d = 128 with P = 128).
 bool tc_bwd_supported(int P, int d, sa_dtype dt) {
   if (dt != SA_BF16 || !tcc::device_is_sm103() || !tc_path_enabled()) return false;
-  return (d == 64 && (P == 128 || P == 256)) || (d == 128 && (P == 128 || P == 256 || P == 512));
+  return (d == 64 && (P == 128 || P == 256)) ||
+         (d == 128 && (P == 128 || P == 256 || P == 512 || P == 1024 || P == 2048));
 }
 
 const char* tc_bwd_name(int P, int d) {
   if (d == 64) return P == 256 ? "tc_bwd_kernel<64,256,full>" : "tc_bwd_kernel<64,128,full>";
+  if (P == 2048) return "tc_bwd_tok_kernel<128,2048>";
+  if (P == 1024) return "tc_bwd_tok_kernel<128,1024>";
   if (P == 512) return "tc_bwd_tok_kernel<128,512>";
   if (P == 256) return "tc_bwd_tok_kernel<128,256>";
   return "tc_bwd_kernel<128,128,full>";
@@ -1073,7 +1076,7 @@ static cudaError_t launch_tok_t(const Args& a, int W, const __nv_bfloat16* gbf, 
 
 }  // namespace tcb
 
-bool tc_bwd_split(int P, int d) { return d == 128 && (P == 256 || P == 512); }
+bool tc_bwd_split(int P, int d) { return d == 128 && (P == 256 || P == 512 || P == 1024 || P == 2048); }
 
 cudaError_t launch_tc_g_bf16(const Args& a, const float* dsk, __nv_bfloat16* gbf, cudaStream_t st) {
   const int64_t n8 = int64_t(a.B) * a.H * a.P * a.d / 8;
@@ -1085,6 +1088,8 @@ cudaError_t launch_tc_bwd_tok(const Args& a, int W, const float* dsk, __nv_bfloa
                               float* Dco, void* dK, void* dV, cudaStream_t st) {
   (void)dsk;
   if (a.N == 0) return cudaSuccess;
+  if (a.P == 2048) return tcb::launch_tok_t<128, 2048>(a, W, gbf, lse, Dco, dK, dV, st);
+  if (a.P == 1024) return tcb::launch_tok_t<128, 1024>(a, W, gbf, lse, Dco, dK, dV, st);
   if (a.P == 512) return tcb::launch_tok_t<128, 512>(a, W, gbf, lse, Dco, dK, dV, st);
   return tcb::launch_tok_t<128, 256>(a, W, gbf, lse, Dco, dK, dV, st);
 }

@@ -456,8 +456,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ------------------------------------------------------------------ lse only
-// Per-token log-sum-exp over all P prototypes, P in chunks of NC <= 256
-// (two TMEM buffers of NC columns alternate over (tile, chunk)).
+// Per-token log-sum-exp over NC * NCH prototypes in chunks of NC <= 256 (two
+// TMEM buffers of NC columns alternate over (tile, chunk)).  With one slice
+// (gridDim.y = 1) these are all P prototypes and the kernel writes lse; with
+// gridDim.y = P / (NC * NCH) slices (P = 1024 or 2048: Q of all prototypes
+// does not fit shared memory) slice y covers prototypes [y NC NCH, (y+1) NC NCH)
+// and writes the token's partial (max of the raw scores, sum of exp2((s - max)
+// scale log2 e)), which combine_lse_kernel folds into lse.
 template <int D, int NC, int NCH>
 struct LseCfg {
   static constexpr int P = NC * NCH;
@@ -478,7 +483,7 @@ struct LseCfg {
 template <int D, int NC, int NCH>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_lse_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ, Args a,
-                  float* __restrict__ lse_out) {
+                  float* __restrict__ lse_out, float2* __restrict__ part_out) {
   using C = LseCfg<D, NC, NCH>;
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -499,6 +504,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
   const int64_t total = tph * a.H;
   const int W = gridDim.x, wk = blockIdx.x;
+  const int NS = gridDim.y, slice = blockIdx.y;  // prototype slices of C::P
+  const int pb = slice * C::P;
   const int64_t tb = range_begin(total, W, wk), te = range_begin(total, W, wk + 1);
   const int ntiles = int(te - tb);
   if (threadIdx.x == 0) {
@@ -541,7 +548,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < NCH; ++c)
 #pragma unroll
             for (int dh = 0; dh < D / 64; ++dh)
-              tma_load_3d(sQ + dh * C::P * 128 + c * NC * 128, &tmQ, q_full, 64 * dh, c * NC, it.qk);
+              tma_load_3d(sQ + dh * C::P * 128 + c * NC * 128, &tmQ, q_full, 64 * dh, pb + c * NC, it.qk);
           prev_h = it.qk;
           ++hc;
         }
@@ -648,7 +655,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (sw == 0 && row < cur.n) {
           const float M = fmaxf(m, o.x);
           const float Z = z * ex2((m - M) * c2) + o.y * ex2((o.x - M) * c2);
-          lse_out[(cur.tok0 + row) * a.H + cur.h] = M * a.scale + logf(Z);
+          const int64_t th = (cur.tok0 + row) * a.H + cur.h;
+          if (NS == 1)
+            lse_out[th] = M * a.scale + logf(Z);
+          else
+            part_out[th * NS + slice] = make_float2(M, Z);
         }
         cur.next();
       }
@@ -695,7 +706,7 @@ static cudaError_t launch_fwd_t(const Args& a, int W, float* sketch, float* lse_
 }
 
 template <int D, int NC, int NCH>
-static cudaError_t launch_lse_t(const Args& a, int W, float* lse_out, cudaStream_t st) {
+static cudaError_t launch_lse_t(const Args& a, int W, float* lse_out, float2* part, cudaStream_t st) {
   using C = LseCfg<D, NC, NCH>;
   CUtensorMap tk, tq;
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, NC))
@@ -703,19 +714,43 @@ static cudaError_t launch_lse_t(const Args& a, int W, float* lse_out, cudaStream
   auto fn = &tc_lse_kernel<D, NC, NCH>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
-  fn<<<W, kThreads, C::SMEM, st>>>(tk, tq, a, lse_out);
+  const int NS = a.P / C::P;
+  dim3 grid(NS > 1 ? (W / NS > 0 ? W / NS : 1) : W, NS);
+  fn<<<grid, kThreads, C::SMEM, st>>>(tk, tq, a, lse_out, part);
   return cudaGetLastError();
+}
+
+// lse[t, h] from the NS per-slice partials (max, sum), folded in slice order.
+__global__ void combine_lse_kernel(const float2* __restrict__ part, int NS, int64_t nth, float scale,
+                                   float* __restrict__ lse, const void* ws) {
+  if (ws_failed(ws)) return;
+  const float c2 = scale * 1.4426950408889634f;
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < nth; i += int64_t(gridDim.x) * blockDim.x) {
+    float2 acc = part[i * NS];
+    for (int k = 1; k < NS; ++k) {
+      const float2 y = part[i * NS + k];
+      const float M = fmaxf(acc.x, y.x);
+      acc = make_float2(M, acc.y * ex2((acc.x - M) * c2) + y.y * ex2((y.x - M) * c2));
+    }
+    lse[i] = acc.x * scale + logf(acc.y);
+  }
 }
 
 }  // namespace tcf
 
-// Shapes served by the tensor-core forward: bf16, d in {64, 128},
-// P in {128, 256} (one CTA holds all prototypes) or P = 512 (lse pass, then
-// two 256-prototype slices).
+// Shapes served by the tensor-core forward: bf16, d in {64, 128}, P in
+// {128, 256} (one CTA holds all prototypes), P = 512 (a cluster pair) or
+// P in {1024, 2048} (sliced lse pass, then 256-prototype slices).
 bool tc_fwd_supported(int P, int d, sa_dtype dt) {
   if (dt != SA_BF16 || (d != 64 && d != 128)) return false;
-  if (P != 128 && P != 256 && P != 512) return false;
+  if (P != 128 && P != 256 && P != 512 && P != 1024 && P != 2048) return false;
   return tcc::device_is_sm103() && tc_path_enabled();
+}
+
+// Prototypes per slice of the lse pass (Q of one slice resident in shared memory).
+int tc_lse_slice(int P, int d) {
+  const int cap = d == 128 ? 512 : 1024;
+  return P < cap ? P : cap;
 }
 
 // By default every supported shape normalises inside the forward kernel:
@@ -723,7 +758,9 @@ bool tc_fwd_supported(int P, int d, sa_dtype dt) {
 // runs P = 512 (and P = 256 with d = 128) as a per-token lse pass followed by
 // 256-prototype slices that take that lse -- the same result computed another
 // way, kept as a cross-check.
-bool tc_fwd_needs_lse_pass_d(int P, int d) { return tc_fwd_sliced_selected() && (P == 512 || (P == 256 && d == 128)); }
+bool tc_fwd_needs_lse_pass_d(int P, int d) {
+  return P >= 1024 || (tc_fwd_sliced_selected() && (P == 512 || (P == 256 && d == 128)));
+}
 
 const char* tc_fwd_name(int P, int d) {
   if (tc_fwd_needs_lse_pass_d(P, d)) return d == 128 ? "tc_fwd_kernel<128,256,sliced>" : "tc_fwd_kernel<64,256,sliced>";
@@ -743,16 +780,24 @@ int tc_fwd_workers(int num_sms, int P, int) {
 cudaError_t launch_tc_lse(const Args& a, float* lse, cudaStream_t st) {
   if (a.N == 0) return cudaSuccess;
   const int W = tcc::device_sm_count();
+  cudaError_t e = cudaErrorInvalidValue;
   if (a.d == 128) {
-    if (a.P == 512) return tcf::launch_lse_t<128, 256, 2>(a, W, lse, st);
-    if (a.P == 256) return tcf::launch_lse_t<128, 256, 1>(a, W, lse, st);
-    if (a.P == 128) return tcf::launch_lse_t<128, 128, 1>(a, W, lse, st);
+    if (a.P >= 512) e = tcf::launch_lse_t<128, 256, 2>(a, W, lse, a.lse_part, st);
+    else if (a.P == 256) e = tcf::launch_lse_t<128, 256, 1>(a, W, lse, a.lse_part, st);
+    else if (a.P == 128) e = tcf::launch_lse_t<128, 128, 1>(a, W, lse, a.lse_part, st);
   } else {
-    if (a.P == 512) return tcf::launch_lse_t<64, 256, 2>(a, W, lse, st);
-    if (a.P == 256) return tcf::launch_lse_t<64, 256, 1>(a, W, lse, st);
-    if (a.P == 128) return tcf::launch_lse_t<64, 128, 1>(a, W, lse, st);
+    if (a.P >= 1024) e = tcf::launch_lse_t<64, 256, 4>(a, W, lse, a.lse_part, st);
+    else if (a.P == 512) e = tcf::launch_lse_t<64, 256, 2>(a, W, lse, a.lse_part, st);
+    else if (a.P == 256) e = tcf::launch_lse_t<64, 256, 1>(a, W, lse, a.lse_part, st);
+    else if (a.P == 128) e = tcf::launch_lse_t<64, 128, 1>(a, W, lse, a.lse_part, st);
   }
-  return cudaErrorInvalidValue;
+  if (e != cudaSuccess) return e;
+  const int NS = a.P / tc_lse_slice(a.P, a.d);
+  if (NS > 1) {
+    tcf::combine_lse_kernel<<<1024, 256, 0, st>>>(a.lse_part, NS, a.N * a.H, a.scale, lse, a.ws);
+    e = cudaGetLastError();
+  }
+  return e;
 }
 
 cudaError_t launch_tc_fwd(const Args& a, int W, float* sketch, float* lse, cudaStream_t st) {

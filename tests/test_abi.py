@@ -45,7 +45,7 @@ def test_status_strings(lib):
 
 def test_workspace_size_rejects_bad_shapes(lib):
     assert binding.sa_workspace_size(1, 10, 1, 0, 64, 1, 0) == 0       # P = 0
-    assert binding.sa_workspace_size(1, 10, 1, 2048, 64, 1, 0) == 0    # P too large
+    assert binding.sa_workspace_size(1, 10, 1, 4096, 64, 1, 0) == 0    # P too large
     assert binding.sa_workspace_size(1, 10, 1, 64, 12, 1, 0) == 0      # d not multiple of 8 (bf16)
     assert binding.sa_workspace_size(0, 10, 1, 64, 64, 1, 0) == 0      # B = 0
     assert binding.sa_workspace_size(1, 2**31, 1, 64, 64, 1, 0) == 0   # N too large

@@ -27,6 +27,9 @@ SHAPES = [
     (96, 32, wl.BF16, 1),
     (200, 128, wl.F32, 1),
     (1024, 64, wl.BF16, 1),
+    (1024, 128, wl.BF16, 1),
+    (2048, 128, wl.BF16, 1),
+    (2048, 64, wl.BF16, 1),
     (1, 8, wl.BF16, 1),
 ]
 
@@ -74,3 +77,10 @@ def test_config5_subbatch(cuda_lib):
     long_u = int(np.nonzero(lens == 1048576)[0][0])
     short_u = [int(u) for u in np.nonzero(lens < 1048576)[0][:40]]
     harness.check_spec(wl.sub_spec(spec, [short_u[0], long_u] + short_u[1:]), bwd=True)
+
+
+def test_large_p_100k_user(cuda_lib):
+    """The paper's final sketch length k = 1K (ablation table: k in {512, 1K, 2K}):
+    one 100K-token user, H=8, d=128, P=1024, Q ~ N(0, 0.02), bf16."""
+    spec = wl.custom([100000], H=8, P=1024, d=128, dtype=wl.BF16, seed=41, q_std=0.02)
+    harness.check_spec(spec, bwd=True)

@@ -9,13 +9,14 @@ from paper_2609_08443_gb300 import binding, workloads as wl
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("P,d", [(128, 64), (256, 64), (128, 128), (256, 128), (512, 128), (512, 64)])
+@pytest.mark.parametrize("P,d", [(128, 64), (256, 64), (128, 128), (256, 128), (512, 128), (512, 64),
+                                 (1024, 128), (1024, 64), (2048, 128)])
 def test_tensor_core_path_matches_cuda_core_path(cuda_lib, P, d):
     spec = wl.custom([700, 0, 128, 129, 3000, 1], H=2, P=P, d=d, dtype=wl.BF16, seed=P * 7 + d)
     host = wl.make_host(spec)
     t = wl.host_to_torch(spec, host, torch.device("cuda"))
     assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, False).startswith("tc_")
-    if (d == 64 and P <= 256) or d == 128:
+    if (d == 64 and P <= 256) or d == 128:  # d = 64 with P >= 512: CUDA-core backward
         assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, True).startswith("tc_")
     tc = harness.gpu_outputs(spec, t, bwd=True)
     binding.sa_select_path(1)

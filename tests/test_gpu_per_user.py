@@ -25,6 +25,7 @@ SHAPES = [
     (256, 64, wl.BF16, 2),    # fused forward, one-CTA backward
     (128, 128, wl.BF16, 2),
     (512, 64, wl.BF16, 1),    # pair forward, CUDA-core backward
+    (1024, 128, wl.BF16, 1),  # sliced lse pass + 4 prototype slices; 8-chunk token side, 8 dQ slices
     (64, 64, wl.F32, 1),      # CUDA cores (fp32)
     (96, 32, wl.BF16, 1),
     (1024, 64, wl.BF16, 1),
