@@ -3,5 +3,5 @@
 Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU baseline /
 reference legs may import this package; the product path never does.
 """
-from .sa_oracle import (affinity, proto_softmax, sa_backward, sa_backward_per_user, sa_forward,  # noqa: F401
-                        sa_forward_per_user)
+from .sa_oracle import (affinity, proto_softmax, sa_backward, sa_backward_per_user, sa_backward_x,  # noqa: F401
+                        sa_forward, sa_forward_per_user, sa_forward_x)

@@ -36,6 +36,12 @@ prototypes Q[b, h] ([B, H, P, d]); the three steps are otherwise unchanged and
 dQ[b, h] = scale * dS K_b collects only user b's tokens
 (``sa_forward_per_user`` / ``sa_backward_per_user``).
 
+Key projection in the step (Sec. 3.1, S = (P W_Q)(X W_K)^T / sqrt(d), sketch
+A X; App. G.3, K = X W_K): the history X serves as the values and, through
+W_K, as the keys.  ``sa_forward_x`` / ``sa_backward_x`` take X [N, H, d] and
+W_K [H, d, d] (per head, k_i = x_i W_K[h]) and return the gradients of X, Q and
+W_K by the chain rule through K = X W_K.
+
 All arithmetic is float64; bf16 inputs arrive already widened exactly.
 Parity pins for both functions live in ``tests/test_oracle.py`` (brute force
 in 50-digit arithmetic, closed forms, invariants, finite differences).
@@ -162,3 +168,28 @@ def sa_backward_per_user(K, V, cu_seqlens, Qu, scale, dO):
             dK[t0:t1, h, :] = scale * (dS.T @ Qu[b, h])
             dQu[b, h] = scale * (dS @ Kb)
     return dK, dV, dQu
+
+
+def _project_keys(X, Wk):
+    """K[:, h, :] = X[:, h, :] @ Wk[h] (Sec. 3.1 / App. G.3, K = X W_K)."""
+    return np.einsum("nhc,hce->nhe", X, Wk)
+
+
+def sa_forward_x(X, cu_seqlens, Q, Wk, scale, with_lse=False):
+    """Sketch with keys projected from the history and the history itself as
+    values: ``sa_forward(X W_K, X, ...)`` (Sec. 3.1)."""
+    X = np.asarray(X, dtype=np.float64)
+    Wk = np.asarray(Wk, dtype=np.float64)
+    return sa_forward(_project_keys(X, Wk), X, cu_seqlens, Q, scale, with_lse=with_lse)
+
+
+def sa_backward_x(X, cu_seqlens, Q, Wk, scale, dO):
+    """Gradients (dX [N,H,d], dQ [H,P,d], dWk [H,d,d]) of L = sum(dO * O) for
+    ``sa_forward_x``: X reaches O twice, as the values and through K = X W_K, so
+    dX = dV + dK W_K^T and dW_K[h] = X[:, h]^T dK[:, h]."""
+    X = np.asarray(X, dtype=np.float64)
+    Wk = np.asarray(Wk, dtype=np.float64)
+    dK, dV, dQ = sa_backward(_project_keys(X, Wk), X, cu_seqlens, Q, scale, dO)
+    dX = dV + np.einsum("nhe,hce->nhc", dK, Wk)
+    dWk = np.einsum("nhc,nhe->hce", X, dK)
+    return dX, dQ, dWk

@@ -389,3 +389,67 @@ def pin_uq_fd_fp64(fwd_uq, bwd_uq, fwd=None, bwd=None):
 
 
 UQ_PINS = [pin_uq_broadcast, pin_uq_users_alone, pin_uq_conservation, pin_uq_fd_fp64]
+
+
+# --------------------------------- key projection in the step (Sec. 3.1)
+# Pins of (fwd_x, bwd_x) with the signatures of oracle.sa_forward_x /
+# oracle.sa_backward_x: X [N, H, d] serves as the values and, through
+# W_K [H, d, d], as the keys.
+
+def _rand_problem_x(seed, lens, H, P, d):
+    X, _, cu, Q, dO = _rand_problem(seed, lens, H, P, d)
+    Wk = _rng(seed + 2000).standard_normal((H, d, d)) / np.sqrt(d)
+    return X, cu, Q, Wk, dO
+
+
+def pin_x_identity_projection(fwd_x, bwd_x, fwd=None, bwd=None):
+    """W_K = I: keys and values are the history itself; the gradient of X is
+    then the sum of the plain oracle's dK and dV."""
+    from oracle import sa_backward, sa_forward
+
+    lens = [5, 0, 8]
+    X, cu, Q, _, dO = _rand_problem_x(41, lens, H=2, P=4, d=3)
+    eye = np.broadcast_to(np.eye(3), (2, 3, 3)).copy()
+    _close(fwd_x(X, cu, Q, eye, 0.8), sa_forward(X, X, cu, Q, 0.8), 1e-12, "sketch, W_K = I")
+    dX, dQ, _ = bwd_x(X, cu, Q, eye, 0.8, dO)
+    dK, dV, dQ1 = sa_backward(X, X, cu, Q, 0.8, dO)
+    _close(dX, dK + dV, 1e-12, "dX, W_K = I")
+    _close(dQ, dQ1, 1e-12, "dQ, W_K = I")
+
+
+def pin_x_folded_prototypes(fwd_x, bwd_x, fwd=None, bwd=None):
+    """S = Q (X W_K)^T = (Q W_K^T) X^T: the sketch equals the plain oracle with
+    prototypes Q W_K^T and K = V = X (associativity of the product)."""
+    from oracle import sa_forward
+
+    lens = [7, 3]
+    X, cu, Q, Wk, _ = _rand_problem_x(42, lens, H=2, P=5, d=4)
+    Qf = np.einsum("hjc,hec->hje", Q, Wk)
+    _close(fwd_x(X, cu, Q, Wk, 0.6), sa_forward(X, X, cu, Qf, 0.6), 1e-12, "sketch with folded prototypes")
+
+
+def pin_x_fd_fp64(fwd_x, bwd_x, fwd=None, bwd=None):
+    """fp64 central differences of the forward for dX, dQ and dW_K."""
+    lens = [6, 4]
+    X, cu, Q, Wk, dO = _rand_problem_x(43, lens, H=2, P=5, d=4)
+    scale = 0.5
+    dX, dQ, dWk = bwd_x(X, cu, Q, Wk, scale, dO)
+    r = _rng(44)
+
+    def loss(X_, Q_, W_):
+        return float(np.sum(dO * fwd_x(X_, cu, Q_, W_, scale)))
+
+    for name, grad in (("X", dX), ("Q", dQ), ("W", dWk)):
+        for _ in range(12):
+            idx = tuple(int(r.integers(0, s)) for s in grad.shape)
+            args = {"X": X.copy(), "Q": Q.copy(), "W": Wk.copy()}
+            h = 1e-6
+            args[name][idx] += h
+            lp = loss(args["X"], args["Q"], args["W"])
+            args[name][idx] -= 2 * h
+            lm = loss(args["X"], args["Q"], args["W"])
+            ref = (lp - lm) / (2 * h)
+            assert abs(grad[idx] - ref) <= 1e-6 * max(1.0, abs(ref)), f"d{name}{idx}"
+
+
+X_PINS = [pin_x_identity_projection, pin_x_folded_prototypes, pin_x_fd_fp64]

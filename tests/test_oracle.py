@@ -3,7 +3,8 @@ import numpy as np
 import pytest
 
 import pins
-from oracle import sa_backward, sa_backward_per_user, sa_forward, sa_forward_per_user
+from oracle import (sa_backward, sa_backward_per_user, sa_backward_x, sa_forward, sa_forward_per_user,
+                    sa_forward_x)
 
 
 @pytest.mark.parametrize("pin", pins.ALL_PINS, ids=lambda p: p.__name__)
@@ -36,3 +37,8 @@ def test_large_scores_do_not_overflow():
 @pytest.mark.parametrize("pin", pins.UQ_PINS, ids=lambda p: p.__name__)
 def test_oracle_per_user_pin(pin):
     pin(sa_forward_per_user, sa_backward_per_user)
+
+
+@pytest.mark.parametrize("pin", pins.X_PINS, ids=lambda p: p.__name__)
+def test_oracle_key_projection_pin(pin):
+    pin(sa_forward_x, sa_backward_x)

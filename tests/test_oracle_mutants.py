@@ -126,3 +126,41 @@ def test_per_user_mutant_is_caught(name):
         except AssertionError:
             caught.append(pin.__name__)
     assert caught, f"no pin catches the planted mistake '{name}'"
+
+
+# --------------------------------- key projection in the step (Sec. 3.1)
+def _x_variant(transpose_wk=False, drop_value_path=False, dwk_transposed=False):
+    def fwd(X, cu, Q, Wk, scale, with_lse=False):
+        W = np.swapaxes(Wk, 1, 2) if transpose_wk else Wk
+        return so.sa_forward_x(X, cu, Q, W, scale, with_lse=with_lse)
+
+    def bwd(X, cu, Q, Wk, scale, dO):
+        W = np.swapaxes(Wk, 1, 2) if transpose_wk else Wk
+        dX, dQ, dW = so.sa_backward_x(X, cu, Q, W, scale, dO)
+        if drop_value_path:
+            dK, dV, _ = so.sa_backward(so._project_keys(np.asarray(X, float), np.asarray(W, float)),
+                                       np.asarray(X, float), cu, Q, scale, dO)
+            dX = dX - dV
+        if dwk_transposed:
+            dW = np.swapaxes(dW, 1, 2)
+        return dX, dQ, dW
+    return fwd, bwd
+
+
+X_MUTANTS = {
+    "keys projected with W_K^T": _x_variant(transpose_wk=True),
+    "dX without the value path": _x_variant(drop_value_path=True),
+    "dW_K transposed": _x_variant(dwk_transposed=True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(X_MUTANTS))
+def test_key_projection_mutant_is_caught(name):
+    fwd, bwd = X_MUTANTS[name]
+    caught = []
+    for pin in pins.X_PINS:
+        try:
+            pin(fwd, bwd)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught, f"no pin catches the planted mistake '{name}'"
