@@ -116,6 +116,29 @@ sa_status sa_sketch_bwd_per_user(const void* K, const void* V, const int32_t* cu
                                  void* dV, float* dQ, void* workspace, size_t ws_bytes,
                                  void* stream);
 
+/* The step with its key projection (Sec. 3.1: S = (P W_Q)(X W_K)^T / sqrt(d),
+ * sketch A X; App. G.3: K = X W_K): the history X serves as the values and,
+ * through W_K, as the keys.
+ *     X  : [N, H, d]  (type `dt`)      Wk : [H, d, d] (type `dt`, k_i = x_i Wk[h])
+ *     Q  : [H, P, d]  (type `dt`, the projected prototypes P W_Q)
+ * Computed as the step with K = V = X and prototypes Q' = Q Wk^T (equal scores:
+ * q_j . (x_i Wk) = (q_j Wk^T) . x_i); no K is formed.  The workspace must hold
+ * sa_workspace_size_x() bytes (the step's own plus Q', and for the backward dK'
+ * and dQ').  Other arguments, results and errors as in sa_sketch_fwd. */
+size_t sa_workspace_size_x(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd);
+sa_status sa_sketch_fwd_x(const void* X, const int32_t* cu_seqlens, int B, int64_t N, const void* Q,
+                          const void* Wk, int H, int P, int d, float scale, sa_dtype dt, float* sketch,
+                          float* lse, void* workspace, size_t ws_bytes, void* stream);
+
+/* Backward of sa_sketch_fwd_x: dX [N,H,d] (type `dt`) = dV + dK W_K^T (X reaches
+ * the sketch as the values and through the keys), dQ [H,P,d] fp32 and
+ * dWk [H,d,d] fp32 = X^T dK per head (chain rule; the paper prints none).  All
+ * outputs are overwritten; `lse` as in sa_sketch_bwd. */
+sa_status sa_sketch_bwd_x(const void* X, const int32_t* cu_seqlens, int B, int64_t N, const void* Q,
+                          const void* Wk, int H, int P, int d, float scale, sa_dtype dt, const float* dsketch,
+                          const float* lse, void* dX, float* dQ, float* dWk, void* workspace, size_t ws_bytes,
+                          void* stream);
+
 /* Allocation-free forward (the paper has no counterpart; this is a library
  * convenience).  For callers that cannot provide a workspace: for example a
  * plugin or custom-operator hook that receives only its input and output

@@ -65,6 +65,13 @@ def load() -> ctypes.CDLL:
     lib.sa_sketch_fwd_per_user.restype = i32
     lib.sa_sketch_bwd_per_user.argtypes = lib.sa_sketch_bwd.argtypes
     lib.sa_sketch_bwd_per_user.restype = i32
+    lib.sa_workspace_size_x.argtypes = [i32, i64, i32, i32, i32, i32, i32]
+    lib.sa_workspace_size_x.restype = sz
+    lib.sa_sketch_fwd_x.argtypes = [vp, vp, i32, i64, vp, vp, i32, i32, i32, f32, i32, vp, vp, vp, sz, vp]
+    lib.sa_sketch_fwd_x.restype = i32
+    lib.sa_sketch_bwd_x.argtypes = [vp, vp, i32, i64, vp, vp, i32, i32, i32, f32, i32, vp, vp, vp, vp, vp, vp,
+                                    sz, vp]
+    lib.sa_sketch_bwd_x.restype = i32
     lib.sa_sketch_fwd_noalloc.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp]
     lib.sa_sketch_fwd_noalloc.restype = i32
     lib.sa_noalloc_scratch_bytes.argtypes = []
@@ -260,6 +267,69 @@ def sa_sketch_fwd_noalloc(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Te
                                    _ptr(sketch), _ptr(lse_out), _stream(K.device))
     _check(st, "sa_sketch_fwd_noalloc")
     return sketch
+
+
+def _validate_x(X, cu, Q, Wk):
+    for name, t in (("X", X), ("Q", Q), ("Wk", Wk), ("cu_seqlens", cu)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    N, H, d = X.shape
+    if Q.dim() != 3 or Q.shape[0] != H or Q.shape[2] != d or tuple(Wk.shape) != (H, d, d):
+        raise ValueError(f"shapes X{tuple(X.shape)} Q{tuple(Q.shape)} Wk{tuple(Wk.shape)}: "
+                         "want X [N,H,d], Q [H,P,d], Wk [H,d,d]")
+    if X.dtype != Q.dtype or X.dtype != Wk.dtype:
+        raise ValueError("X, Q and Wk must share one dtype")
+    if cu.dtype != torch.int32 or cu.dim() != 1 or cu.numel() < 2:
+        raise ValueError("cu_seqlens must be int32 [B+1]")
+
+
+def sa_sketch_fwd_x(X: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor, Wk: torch.Tensor,
+                    scale: Optional[float] = None, want_lse: bool = False, ws: Optional[torch.Tensor] = None):
+    """Sketch with keys X Wk[h] and values X (Sec. 3.1): [B,H,P,d] fp32 (and lse)."""
+    lib = load()
+    _validate_x(X, cu_seqlens, Q, Wk)
+    N, H, d = X.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    dt = _dt(X)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    sketch = torch.empty((B, H, P, d), dtype=torch.float32, device=X.device)
+    lse = torch.empty((N, H), dtype=torch.float32, device=X.device) if want_lse else None
+    need = lib.sa_workspace_size_x(B, N, H, P, d, dt, 0)
+    if need == 0:
+        raise SketchError(2, "sa_workspace_size_x")
+    w = ws if ws is not None else workspace(need, X.device)
+    st = lib.sa_sketch_fwd_x(_ptr(X), _ptr(cu_seqlens), B, N, _ptr(Q), _ptr(Wk), H, P, d, scale, dt,
+                             _ptr(sketch), _ptr(lse), _ptr(w), w.numel(), _stream(X.device))
+    _check(st, "sa_sketch_fwd_x")
+    return (sketch, lse) if want_lse else sketch
+
+
+def sa_sketch_bwd_x(X: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor, Wk: torch.Tensor,
+                    dsketch: torch.Tensor, scale: Optional[float] = None, lse: Optional[torch.Tensor] = None,
+                    ws: Optional[torch.Tensor] = None):
+    """(dX like X, dQ [H,P,d] fp32, dWk [H,d,d] fp32) for ``sa_sketch_fwd_x``."""
+    lib = load()
+    _validate_x(X, cu_seqlens, Q, Wk)
+    N, H, d = X.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    if dsketch.shape != (B, H, P, d) or dsketch.dtype != torch.float32 or not dsketch.is_contiguous():
+        raise ValueError("dsketch must be contiguous fp32 [B,H,P,d]")
+    dt = _dt(X)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    dX = torch.empty_like(X)
+    dQ = torch.empty((H, P, d), dtype=torch.float32, device=X.device)
+    dWk = torch.empty((H, d, d), dtype=torch.float32, device=X.device)
+    need = lib.sa_workspace_size_x(B, N, H, P, d, dt, 1)
+    if need == 0:
+        raise SketchError(2, "sa_workspace_size_x")
+    w = ws if ws is not None else workspace(need, X.device)
+    st = lib.sa_sketch_bwd_x(_ptr(X), _ptr(cu_seqlens), B, N, _ptr(Q), _ptr(Wk), H, P, d, scale, dt,
+                             _ptr(dsketch), _ptr(lse), _ptr(dX), _ptr(dQ), _ptr(dWk), _ptr(w), w.numel(),
+                             _stream(X.device))
+    _check(st, "sa_sketch_bwd_x")
+    return dX, dQ, dWk
 
 
 def sa_noalloc_scratch_bytes() -> int:

@@ -352,6 +352,57 @@ sa_status sa_sketch_bwd_per_user(const void* K, const void* V, const int32_t* cu
                   stream, 1);
 }
 
+// ------------------------------------------- key projection (Sec. 3.1, K = X W_K)
+static size_t x_elem(sa_dtype dt) { return dt == SA_BF16 ? 2 : 4; }
+
+// Extra workspace of the X entry points, after the step's own: Q' = Q W_K^T
+// [H,P,d] (dt); for the backward also dK' [N,H,d] (dt) and dQ' [H,P,d] (fp32).
+static size_t x_extra(int64_t N, int H, int P, int d, sa_dtype dt, bool bwd) {
+  size_t b = sa::align256(size_t(H) * P * d * x_elem(dt));
+  if (bwd) b += sa::align256(size_t(N) * H * d * x_elem(dt)) + sa::align256(size_t(H) * P * d * 4);
+  return b;
+}
+
+size_t sa_workspace_size_x(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd) {
+  const size_t base = sa_workspace_size(B, N, H, P, d, dt, bwd);
+  return base == 0 ? 0 : base + x_extra(N, H, P, d, dt, bwd != 0);
+}
+
+sa_status sa_sketch_fwd_x(const void* X, const int32_t* cu_seqlens, int B, int64_t N, const void* Q,
+                          const void* Wk, int H, int P, int d, float scale, sa_dtype dt, float* sketch, float* lse,
+                          void* workspace, size_t ws_bytes, void* stream) {
+  if (!Q || !Wk || !workspace || (N > 0 && !X)) return SA_ERR_INVALID_ARG;
+  const size_t base = sa_workspace_size(B, N, H, P, d, dt, 0);
+  if (base == 0) return shape_ok(B, N, H, P, d, dt) ? SA_ERR_INVALID_ARG : SA_ERR_UNSUPPORTED;
+  if (ws_bytes < base + x_extra(N, H, P, d, dt, false)) return SA_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 || !aligned16(Wk)) return SA_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void* Qf = static_cast<char*>(workspace) + base;
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_fold_wk(Q, Wk, H, P, d, dt, Qf, st); }));
+  return fwd_impl(X, X, cu_seqlens, B, N, Qf, H, P, d, scale, dt, sketch, lse, workspace, base, stream, 0);
+}
+
+sa_status sa_sketch_bwd_x(const void* X, const int32_t* cu_seqlens, int B, int64_t N, const void* Q,
+                          const void* Wk, int H, int P, int d, float scale, sa_dtype dt, const float* dsketch,
+                          const float* lse, void* dX, float* dQ, float* dWk, void* workspace, size_t ws_bytes,
+                          void* stream) {
+  if (!Q || !Wk || !dQ || !dWk || !workspace || (N > 0 && (!X || !dX))) return SA_ERR_INVALID_ARG;
+  const size_t base = sa_workspace_size(B, N, H, P, d, dt, 1);
+  if (base == 0) return shape_ok(B, N, H, P, d, dt) ? SA_ERR_INVALID_ARG : SA_ERR_UNSUPPORTED;
+  if (ws_bytes < base + x_extra(N, H, P, d, dt, true)) return SA_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 || !aligned16(Wk)) return SA_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* Qf = static_cast<char*>(workspace) + base;
+  char* dKf = Qf + sa::align256(size_t(H) * P * d * x_elem(dt));
+  float* dQf = reinterpret_cast<float*>(dKf + sa::align256(size_t(N) * H * d * x_elem(dt)));
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_fold_wk(Q, Wk, H, P, d, dt, Qf, st); }));
+  // the step with K = V = X and prototypes Q': dK' to the workspace, dV into dX
+  SA_TRY(bwd_impl(X, X, cu_seqlens, B, N, Qf, H, P, d, scale, dt, dsketch, lse, N > 0 ? dKf : nullptr, dX, dQf,
+                  workspace, base, stream, 0));
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_add_into(dX, dKf, N * H * int64_t(d), dt, st); }));
+  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_wk_grads(dQf, Q, Wk, H, P, d, dt, dQ, dWk, st); });
+}
+
 sa_status sa_get_device_error(const void* workspace, void* stream) {
   if (!workspace) return SA_ERR_INVALID_ARG;
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return SA_ERR_CUDA;

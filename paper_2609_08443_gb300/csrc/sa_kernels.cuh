@@ -33,6 +33,13 @@ cudaError_t launch_plan(const Args& a, int T, cudaStream_t st);
 cudaError_t launch_finalize_sketch(const Args& a, int W, float* sketch, cudaStream_t st);
 cudaError_t launch_finalize_dq(const Args& a, int W, float* dQ, cudaStream_t st);
 
+// key projection folded into the prototypes (sa_xproj.cu)
+cudaError_t launch_fold_wk(const void* Q, const void* Wk, int H, int P, int d, sa_dtype dt, void* Qf,
+                           cudaStream_t st);
+cudaError_t launch_add_into(void* dX, const void* dKf, int64_t n, sa_dtype dt, cudaStream_t st);
+cudaError_t launch_wk_grads(const float* dQf, const void* Q, const void* Wk, int H, int P, int d, sa_dtype dt,
+                            float* dQ, float* dWk, cudaStream_t st);
+
 // CUDA-core path (sa_simt.cu)
 int simt_tile_tokens();
 int simt_workers(int num_sms, int P);
