@@ -42,6 +42,12 @@ W_K, as the keys.  ``sa_forward_x`` / ``sa_backward_x`` take X [N, H, d] and
 W_K [H, d, d] (per head, k_i = x_i W_K[h]) and return the gradients of X, Q and
 W_K by the chain rule through K = X W_K.
 
+Token-wise ("vanilla") normalisation, the comparison of Sec. 5.1 and App. C:
+the same scores normalised over the user's tokens instead of the prototypes,
+A[j, :] = softmax over i of S[j, i] (weights p(i | j), each prototype
+selecting tokens), sketch = A V_b (``sa_forward_tokenwise`` /
+``sa_backward_tokenwise``; the softmax Jacobian then runs along the token axis).
+
 All arithmetic is float64; bf16 inputs arrive already widened exactly.
 Parity pins for both functions live in ``tests/test_oracle.py`` (brute force
 in 50-digit arithmetic, closed forms, invariants, finite differences).
@@ -193,3 +199,59 @@ def sa_backward_x(X, cu_seqlens, Q, Wk, scale, dO):
     dX = dV + np.einsum("nhe,hce->nhc", dK, Wk)
     dWk = np.einsum("nhc,nhe->hce", X, dK)
     return dX, dQ, dWk
+
+
+def token_softmax(S):
+    """Softmax along axis 1 (the token axis) of a P x L score matrix, max
+    subtracted per row (Sec. 5.1 / App. C: weights p(i | j))."""
+    m = S.max(axis=1, keepdims=True)
+    e = np.exp(S - m)
+    return e / e.sum(axis=1, keepdims=True)
+
+
+def sa_forward_tokenwise(K, V, cu_seqlens, Q, scale, with_lse=False):
+    """Sketch O[B, H, P, d] under token-wise normalisation (and, with
+    ``with_lse``, the per-prototype log-sum-exp over the user's tokens,
+    lse_tok[B, H, P]).  A user with no tokens gets O = 0 and lse_tok = -inf."""
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Q = np.asarray(Q, dtype=np.float64)
+    H, P, d = Q.shape
+    sl = _user_slices(cu_seqlens)
+    O = np.zeros((len(sl), H, P, d))
+    lse = np.full((len(sl), H, P), -np.inf)
+    for b, (t0, t1) in enumerate(sl):
+        if t1 == t0:
+            continue
+        for h in range(H):
+            S = affinity(Q[h], K[t0:t1, h, :], scale)
+            O[b, h] = token_softmax(S) @ V[t0:t1, h, :]
+            m = S.max(axis=1)
+            lse[b, h] = m + np.log(np.exp(S - m[:, None]).sum(axis=1))
+    return (O, lse) if with_lse else O
+
+
+def sa_backward_tokenwise(K, V, cu_seqlens, Q, scale, dO):
+    """Gradients (dK [N,H,d], dV [N,H,d], dQ [H,P,d]) of L = sum(dO * O) for
+    ``sa_forward_tokenwise``: dS = A * (dA - rowsum(A * dA)) (softmax Jacobian
+    along the token axis); dQ sums over all users (shared prototypes)."""
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Q = np.asarray(Q, dtype=np.float64)
+    dO = np.asarray(dO, dtype=np.float64)
+    H, P, d = Q.shape
+    dK = np.zeros_like(K)
+    dV = np.zeros_like(V)
+    dQ = np.zeros_like(Q)
+    for b, (t0, t1) in enumerate(_user_slices(cu_seqlens)):
+        if t1 == t0:
+            continue
+        for h in range(H):
+            Kb, Vb, G = K[t0:t1, h, :], V[t0:t1, h, :], dO[b, h]
+            A = token_softmax(affinity(Q[h], Kb, scale))
+            dV[t0:t1, h, :] = A.T @ G
+            dA = G @ Vb.T
+            dS = A * (dA - (A * dA).sum(axis=1, keepdims=True))
+            dK[t0:t1, h, :] = scale * (dS.T @ Q[h])
+            dQ[h] += scale * (dS @ Kb)
+    return dK, dV, dQ

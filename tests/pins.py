@@ -453,3 +453,95 @@ def pin_x_fd_fp64(fwd_x, bwd_x, fwd=None, bwd=None):
 
 
 X_PINS = [pin_x_identity_projection, pin_x_folded_prototypes, pin_x_fd_fp64]
+
+
+# ------------------------- token-wise ("vanilla") normalisation (Sec. 5.1)
+# Pins of (fwd_tw, bwd_tw) with the signatures of oracle.sa_forward_tokenwise /
+# oracle.sa_backward_tokenwise (weights normalised over each user's tokens).
+
+def pin_tw_bruteforce(fwd_tw, bwd_tw=None, fwd=None, bwd=None):
+    """50-digit plain loops of A[j, i] = exp(S[j, i]) / sum_i' exp(S[j, i']),
+    O = A V, no stabilising shift."""
+    import mpmath as mp
+
+    mp.mp.dps = 50
+    lens = [3, 0, 2]
+    K, V, cu, Q, _ = _rand_problem(51, lens, H=2, P=3, d=2)
+    scale = 0.9
+    O = fwd_tw(K, V, cu, Q, scale)
+    for b in range(len(lens)):
+        t0, t1 = int(cu[b]), int(cu[b + 1])
+        for h in range(2):
+            for j in range(3):
+                s = [mp.mpf(scale) * mp.fsum(mp.mpf(Q[h, j, c]) * mp.mpf(K[i, h, c]) for c in range(2))
+                     for i in range(t0, t1)]
+                z = mp.fsum(mp.exp(x) for x in s)
+                for c in range(2):
+                    ref = mp.fsum(mp.exp(s[i - t0]) / z * mp.mpf(V[i, h, c]) for i in range(t0, t1)) if s else 0
+                    assert abs(O[b, h, j, c] - float(ref)) <= 1e-12 * max(1.0, abs(float(ref))), (b, h, j, c)
+
+
+def pin_tw_rows_sum_to_one(fwd_tw, bwd_tw=None, fwd=None, bwd=None):
+    """V = 1: every sketch entry of a non-empty user is 1 (sum_i A[j, i] = 1)."""
+    lens = [4, 0, 9]
+    K, V, cu, Q, _ = _rand_problem(52, lens, H=2, P=5, d=3)
+    O = fwd_tw(K, np.ones_like(V), cu, Q, 0.7)
+    _close(O[0], np.ones((2, 5, 3)), 1e-12, "user 0")
+    _close(O[2], np.ones((2, 5, 3)), 1e-12, "user 2")
+    assert np.all(O[1] == 0), "an empty user has a zero sketch"
+
+
+def pin_tw_closed_forms(fwd_tw, bwd_tw=None, fwd=None, bwd=None):
+    """One token: O[j] = v_1 for every prototype.  Equal keys: O[j] is the mean
+    of the user's values.  A huge scale: O[j] = v at arg max_i S[j, i]."""
+    r = _rng(53)
+    Q = r.standard_normal((1, 4, 3))
+    K1, V1 = r.standard_normal((1, 1, 3)), r.standard_normal((1, 1, 3))
+    _close(fwd_tw(K1, V1, np.array([0, 1]), Q, 0.5)[0, 0], np.repeat(V1[0], 4, axis=0), 1e-12, "one token")
+    Ke = np.repeat(r.standard_normal((1, 1, 3)), 6, axis=0)
+    Ve = r.standard_normal((6, 1, 3))
+    _close(fwd_tw(Ke, Ve, np.array([0, 6]), Q, 0.5)[0, 0], np.repeat(Ve.mean(axis=0), 4, axis=0), 1e-12, "equal keys")
+    Kh, Vh = r.standard_normal((7, 1, 3)), r.standard_normal((7, 1, 3))
+    O = fwd_tw(Kh, Vh, np.array([0, 7]), Q, 1e4)[0, 0]
+    arg = np.argmax(Q[0] @ Kh[:, 0, :].T, axis=1)
+    _close(O, Vh[arg, 0, :], 1e-9, "hard selection")
+
+
+def pin_tw_token_order(fwd_tw, bwd_tw, fwd=None, bwd=None):
+    """Permuting a user's tokens permutes dK, dV and changes nothing else."""
+    lens = [8]
+    K, V, cu, Q, dO = _rand_problem(54, lens, H=2, P=4, d=3)
+    perm = _rng(55).permutation(8)
+    _close(fwd_tw(K[perm], V[perm], cu, Q, 0.6), fwd_tw(K, V, cu, Q, 0.6), 1e-12, "sketch under permutation")
+    dK, dV, dQ = bwd_tw(K, V, cu, Q, 0.6, dO)
+    dKp, dVp, dQp = bwd_tw(K[perm], V[perm], cu, Q, 0.6, dO)
+    _close(dKp, dK[perm], 1e-12, "dK under permutation")
+    _close(dVp, dV[perm], 1e-12, "dV under permutation")
+    _close(dQp, dQ, 1e-12, "dQ under permutation")
+
+
+def pin_tw_fd_fp64(fwd_tw, bwd_tw, fwd=None, bwd=None):
+    """fp64 central differences for dK, dV, dQ."""
+    lens = [7, 0, 5]
+    K, V, cu, Q, dO = _rand_problem(56, lens, H=2, P=6, d=4)
+    scale = 0.5
+    dK, dV, dQ = bwd_tw(K, V, cu, Q, scale, dO)
+    r = _rng(57)
+
+    def loss(K_, V_, Q_):
+        return float(np.sum(dO * fwd_tw(K_, V_, cu, Q_, scale)))
+
+    for name, grad in (("K", dK), ("V", dV), ("Q", dQ)):
+        for _ in range(12):
+            idx = tuple(int(r.integers(0, s)) for s in grad.shape)
+            args = {"K": K.copy(), "V": V.copy(), "Q": Q.copy()}
+            h = 1e-6
+            args[name][idx] += h
+            lp = loss(args["K"], args["V"], args["Q"])
+            args[name][idx] -= 2 * h
+            lm = loss(args["K"], args["V"], args["Q"])
+            ref = (lp - lm) / (2 * h)
+            assert abs(grad[idx] - ref) <= 1e-6 * max(1.0, abs(ref)), f"d{name}{idx}"
+
+
+TW_PINS = [pin_tw_bruteforce, pin_tw_rows_sum_to_one, pin_tw_closed_forms, pin_tw_token_order, pin_tw_fd_fp64]

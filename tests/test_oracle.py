@@ -3,8 +3,8 @@ import numpy as np
 import pytest
 
 import pins
-from oracle import (sa_backward, sa_backward_per_user, sa_backward_x, sa_forward, sa_forward_per_user,
-                    sa_forward_x)
+from oracle import (sa_backward, sa_backward_per_user, sa_backward_tokenwise, sa_backward_x, sa_forward,
+                    sa_forward_per_user, sa_forward_tokenwise, sa_forward_x)
 
 
 @pytest.mark.parametrize("pin", pins.ALL_PINS, ids=lambda p: p.__name__)
@@ -42,3 +42,10 @@ def test_oracle_per_user_pin(pin):
 @pytest.mark.parametrize("pin", pins.X_PINS, ids=lambda p: p.__name__)
 def test_oracle_key_projection_pin(pin):
     pin(sa_forward_x, sa_backward_x)
+
+
+@pytest.mark.parametrize("pin", pins.TW_PINS, ids=lambda p: p.__name__)
+def test_oracle_tokenwise_pin(pin):
+    if pin.__name__.endswith("bruteforce"):
+        pytest.importorskip("mpmath")
+    pin(sa_forward_tokenwise, sa_backward_tokenwise)

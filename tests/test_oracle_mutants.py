@@ -164,3 +164,51 @@ def test_key_projection_mutant_is_caught(name):
         except AssertionError:
             caught.append(pin.__name__)
     assert caught, f"no pin catches the planted mistake '{name}'"
+
+
+# ------------------------- token-wise ("vanilla") normalisation (Sec. 5.1)
+def _tw_variant(proto_axis=False, drop_d=False, dv_from_g_t=False):
+    def fwd(K, V, cu, Q, scale, with_lse=False):
+        if proto_axis:
+            return so.sa_forward(K, V, cu, Q, scale, with_lse=with_lse)
+        return so.sa_forward_tokenwise(K, V, cu, Q, scale, with_lse=with_lse)
+
+    def bwd(K, V, cu, Q, scale, dO):
+        K = np.asarray(K, float); V = np.asarray(V, float); Q = np.asarray(Q, float); dO = np.asarray(dO, float)
+        H, P, d = Q.shape
+        dK = np.zeros_like(K); dV = np.zeros_like(V); dQ = np.zeros_like(Q)
+        for b, (t0, t1) in enumerate(so._user_slices(cu)):
+            if t1 == t0:
+                continue
+            for h in range(H):
+                Kb, Vb, G = K[t0:t1, h], V[t0:t1, h], dO[b, h]
+                A = so.token_softmax(scale * (Q[h] @ Kb.T))
+                dV[t0:t1, h] = (A.T @ G) if not dv_from_g_t else (A.T @ G[::-1])
+                dA = G @ Vb.T
+                Dv = 0.0 if drop_d else (A * dA).sum(axis=1, keepdims=True)
+                dS = A * (dA - Dv)
+                dK[t0:t1, h] = scale * (dS.T @ Q[h])
+                dQ[h] += scale * (dS @ Kb)
+        return dK, dV, dQ
+    return fwd, bwd
+
+
+TW_MUTANTS = {
+    "normalised over prototypes": _tw_variant(proto_axis=True),
+    "dS without the row term": _tw_variant(drop_d=True),
+    "dV with prototypes reversed": _tw_variant(dv_from_g_t=True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(TW_MUTANTS))
+def test_tokenwise_mutant_is_caught(name):
+    fwd, bwd = TW_MUTANTS[name]
+    caught = []
+    for pin in pins.TW_PINS:
+        if pin.__name__.endswith("bruteforce"):
+            pytest.importorskip("mpmath")
+        try:
+            pin(fwd, bwd)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught, f"no pin catches the planted mistake '{name}'"
