@@ -139,6 +139,35 @@ sa_status sa_sketch_bwd_x(const void* X, const int32_t* cu_seqlens, int B, int64
                           const float* lse, void* dX, float* dQ, float* dWk, void* workspace, size_t ws_bytes,
                           void* stream);
 
+/* Token-wise ("vanilla") normalisation, the comparison of Sec. 5.1 and App. C:
+ * the same scores normalised over each user's tokens instead of the prototypes,
+ *     A[j, :]      = softmax over i of S[j, i]     (weights p(i | j): every
+ *                    prototype spreads unit mass over the user's tokens)
+ *     sketch[b, h] = A V_b                          (P x d)
+ *     lse_tok      : [B, H, P] fp32, log sum_i exp(S[j, i]) per user, head and
+ *                    prototype (-inf for a user with L_b = 0, whose sketch is 0)
+ * `lse_tok` may be NULL.  Shared prototypes Q [H, P, d] only.  CUDA-core
+ * kernels (fp32 arithmetic) for both dtypes.  The workspace must hold
+ * sa_workspace_size_tokenwise() bytes; everything else (layouts, ownership,
+ * errors, determinism) as in sa_sketch_fwd. */
+size_t sa_workspace_size_tokenwise(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd);
+sa_status sa_sketch_fwd_tokenwise(const void* K, const void* V, const int32_t* cu_seqlens, int B,
+                                  int64_t N, const void* Q, int H, int P, int d, float scale,
+                                  sa_dtype dt, float* sketch, float* lse_tok, void* workspace,
+                                  size_t ws_bytes, void* stream);
+
+/* Backward of sa_sketch_fwd_tokenwise for dsketch G [B,H,P,d] (chain rule; the
+ * paper prints none), with D_j = G_j . sketch_j per user and head:
+ *     dV_i = sum_j A[j,i] G_j,    dS[j,i] = A[j,i] (G_j . v_i - D_j),
+ *     dK_i = scale sum_j dS[j,i] Q_j,    dQ[h] = scale sum_b sum_i dS[:,i] K_b[i,h].
+ * `sketch` and `lse_tok` are the forward's outputs; when either is NULL both are
+ * recomputed.  dK, dV have type `dt`, dQ is fp32; all fully overwritten. */
+sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* cu_seqlens, int B,
+                                  int64_t N, const void* Q, int H, int P, int d, float scale,
+                                  sa_dtype dt, const float* sketch, const float* lse_tok,
+                                  const float* dsketch, void* dK, void* dV, float* dQ,
+                                  void* workspace, size_t ws_bytes, void* stream);
+
 /* Allocation-free forward (the paper has no counterpart; this is a library
  * convenience).  For callers that cannot provide a workspace: for example a
  * plugin or custom-operator hook that receives only its input and output

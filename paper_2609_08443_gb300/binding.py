@@ -76,6 +76,13 @@ def load() -> ctypes.CDLL:
     lib.sa_sketch_fwd_noalloc.restype = i32
     lib.sa_noalloc_scratch_bytes.argtypes = []
     lib.sa_noalloc_scratch_bytes.restype = sz
+    lib.sa_workspace_size_tokenwise.argtypes = [i32, i64, i32, i32, i32, i32, i32]
+    lib.sa_workspace_size_tokenwise.restype = sz
+    lib.sa_sketch_fwd_tokenwise.argtypes = lib.sa_sketch_fwd.argtypes
+    lib.sa_sketch_fwd_tokenwise.restype = i32
+    lib.sa_sketch_bwd_tokenwise.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp, vp, vp,
+                                            vp, vp, sz, vp]
+    lib.sa_sketch_bwd_tokenwise.restype = i32
     lib.sa_plan_host.argtypes = [vp, i32, i32, i32, i32, vp]
     lib.sa_plan_host.restype = i32
     _lib = lib
@@ -330,6 +337,64 @@ def sa_sketch_bwd_x(X: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor, 
                              _stream(X.device))
     _check(st, "sa_sketch_bwd_x")
     return dX, dQ, dWk
+
+
+def sa_sketch_fwd_tokenwise(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
+                            scale: Optional[float] = None, want_lse: bool = False,
+                            ws: Optional[torch.Tensor] = None):
+    """Token-wise normalisation (Sec. 5.1, App. C): sketch [B,H,P,d] fp32 with
+    weights softmax over each user's tokens per prototype (and lse_tok [B,H,P])."""
+    lib = load()
+    _validate(K, V, cu_seqlens, Q)
+    if Q.dim() != 3:
+        raise ValueError("the token-wise variant takes shared prototypes Q [H,P,d]")
+    N, H, d = K.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    dt = _dt(K)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    sketch = torch.empty((B, H, P, d), dtype=torch.float32, device=K.device)
+    lse = torch.empty((B, H, P), dtype=torch.float32, device=K.device) if want_lse else None
+    need = lib.sa_workspace_size_tokenwise(B, N, H, P, d, dt, 0)
+    if need == 0:
+        raise SketchError(2, "sa_workspace_size_tokenwise")
+    w = ws if ws is not None else workspace(need, K.device)
+    st = lib.sa_sketch_fwd_tokenwise(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
+                                     _ptr(sketch), _ptr(lse), _ptr(w), w.numel(), _stream(K.device))
+    _check(st, "sa_sketch_fwd_tokenwise")
+    return (sketch, lse) if want_lse else sketch
+
+
+def sa_sketch_bwd_tokenwise(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
+                            dsketch: torch.Tensor, scale: Optional[float] = None,
+                            sketch: Optional[torch.Tensor] = None, lse: Optional[torch.Tensor] = None,
+                            ws: Optional[torch.Tensor] = None):
+    """(dK, dV, dQ [H,P,d] fp32) of ``sa_sketch_fwd_tokenwise``; ``sketch`` and
+    ``lse`` are the forward's outputs (recomputed when either is missing)."""
+    lib = load()
+    _validate(K, V, cu_seqlens, Q)
+    if Q.dim() != 3:
+        raise ValueError("the token-wise variant takes shared prototypes Q [H,P,d]")
+    N, H, d = K.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    for name, t, shape in (("dsketch", dsketch, (B, H, P, d)), ("sketch", sketch, (B, H, P, d)),
+                           ("lse", lse, (B, H, P))):
+        if t is not None and (tuple(t.shape) != shape or t.dtype != torch.float32 or not t.is_contiguous()):
+            raise ValueError(f"{name} must be contiguous fp32 {list(shape)}")
+    dt = _dt(K)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    dK, dV = torch.empty_like(K), torch.empty_like(V)
+    dQ = torch.empty((H, P, d), dtype=torch.float32, device=K.device)
+    need = lib.sa_workspace_size_tokenwise(B, N, H, P, d, dt, 1)
+    if need == 0:
+        raise SketchError(2, "sa_workspace_size_tokenwise")
+    w = ws if ws is not None else workspace(need, K.device)
+    st = lib.sa_sketch_bwd_tokenwise(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
+                                     _ptr(sketch), _ptr(lse), _ptr(dsketch), _ptr(dK), _ptr(dV), _ptr(dQ),
+                                     _ptr(w), w.numel(), _stream(K.device))
+    _check(st, "sa_sketch_bwd_tokenwise")
+    return dK, dV, dQ
 
 
 def sa_noalloc_scratch_bytes() -> int:

@@ -118,9 +118,9 @@ Plan make_plan(int B, int64_t N, int H, int P, int d, sa_dtype dt, bool bwd) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-sa_status check_common(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q,
-                       int H, int P, int d, float scale, sa_dtype dt, const void* ws, size_t ws_bytes,
-                       bool bwd, Plan* plan) {
+// Checks every entry point applies before choosing kernels.
+sa_status check_args(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q, int H, int P,
+                     int d, float scale, sa_dtype dt, const void* ws) {
   if (!cu || !Q || !ws) return SA_ERR_INVALID_ARG;
   if (N > 0 && (!K || !V)) return SA_ERR_INVALID_ARG;
   if (!std::isfinite(scale)) return SA_ERR_INVALID_ARG;
@@ -128,6 +128,13 @@ sa_status check_common(const void* K, const void* V, const int32_t* cu, int B, i
   if (!shape_ok(B, N, H, P, d, dt)) return SA_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return SA_ERR_INVALID_ARG;
   if ((K && !aligned16(K)) || (V && !aligned16(V)) || !aligned16(Q)) return SA_ERR_INVALID_ARG;
+  return SA_OK;
+}
+
+sa_status check_common(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q,
+                       int H, int P, int d, float scale, sa_dtype dt, const void* ws, size_t ws_bytes,
+                       bool bwd, Plan* plan) {
+  SA_TRY(check_args(K, V, cu, B, N, Q, H, P, d, scale, dt, ws));
   *plan = make_plan(B, N, H, P, d, dt, bwd);
   if (ws_bytes < plan->lay.total) return SA_ERR_WORKSPACE;
   return SA_OK;
@@ -401,6 +408,106 @@ sa_status sa_sketch_bwd_x(const void* X, const int32_t* cu_seqlens, int B, int64
                   workspace, base, stream, 0));
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_add_into(dX, dKf, N * H * int64_t(d), dt, st); }));
   return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_wk_grads(dQf, Q, Wk, H, P, d, dt, dQ, dWk, st); });
+}
+
+// ------------------------------ token-wise normalisation (Sec. 5.1, App. C)
+namespace {
+
+// Workspace of the token-wise entry points (CUDA-core kernels, 32-token tiles):
+// header | tile prefix | cut-segment pieces [W][2][P][d] | dQ pieces [W][H][P][d]
+// (bwd) | piece statistics float2 [W][2][P] | lse_tok [B][H][P] | D [B][H][P] (bwd)
+// | sketch recomputed by the backward [B][H][P][d] (bwd).
+struct TwLayout {
+  sa::WsLayout base;
+  size_t stat_part, lse_tok, dcoef, sketch, total;
+  int W;
+};
+
+TwLayout tw_layout(int B, int H, int P, int d, bool bwd) {
+  TwLayout t{};
+  t.W = sa::simt_workers(device_sms() > 0 ? device_sms() : 1, P);
+  sa::WsLayout& L = t.base;
+  size_t off = sizeof(sa::WsHeader);
+  L.tile_prefix = off;
+  off = sa::align256(off + sizeof(int64_t) * size_t(B + 1));
+  L.partial = off;
+  off = sa::align256(off + sizeof(float) * size_t(t.W) * 2 * P * d);
+  L.dq_partial = off;
+  if (bwd) off = sa::align256(off + sizeof(float) * size_t(t.W) * H * P * d);
+  t.stat_part = off;
+  off = sa::align256(off + sizeof(float2) * size_t(t.W) * 2 * P);
+  t.lse_tok = off;
+  off = sa::align256(off + sizeof(float) * size_t(B) * H * P);
+  t.dcoef = off;
+  t.sketch = off;
+  if (bwd) {
+    off = sa::align256(off + sizeof(float) * size_t(B) * H * P);
+    t.sketch = off;
+    off = sa::align256(off + sizeof(float) * size_t(B) * H * P * d);
+  }
+  L.lse = L.dcoef = L.gbf = L.lse_part = off;  // unused on this path
+  L.total = t.total = off;
+  return t;
+}
+
+sa_status tw_check(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q, int H, int P,
+                   int d, float scale, sa_dtype dt, const void* ws, size_t ws_bytes, bool bwd, TwLayout* lay) {
+  SA_TRY(check_args(K, V, cu, B, N, Q, H, P, d, scale, dt, ws));
+  *lay = tw_layout(B, H, P, d, bwd);
+  return ws_bytes < lay->total ? SA_ERR_WORKSPACE : SA_OK;
+}
+
+// Plan, online-softmax sweep, merge of cut segments: sketch and lse_tok.
+sa_status tw_forward(const sa::Args& a, const TwLayout& lay, float* sketch, float* lse_tok, cudaStream_t st) {
+  float2* stat = reinterpret_cast<float2*>(static_cast<char*>(a.ws) + lay.stat_part);
+  SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_tw_fwd(a, lay.W, sketch, lse_tok, stat, st); }));
+  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tw_finalize(a, lay.W, stat, sketch, lse_tok, st); });
+}
+
+}  // namespace
+
+size_t sa_workspace_size_tokenwise(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd) {
+  if (!shape_ok(B, N, H, P, d, dt)) return 0;
+  return tw_layout(B, H, P, d, bwd != 0).total;
+}
+
+sa_status sa_sketch_fwd_tokenwise(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                                  const void* Q, int H, int P, int d, float scale, sa_dtype dt, float* sketch,
+                                  float* lse_tok, void* workspace, size_t ws_bytes, void* stream) {
+  if (!sketch) return SA_ERR_INVALID_ARG;
+  TwLayout lay;
+  SA_TRY(tw_check(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, false, &lay));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, lay.base);
+  if (!lse_tok) lse_tok = reinterpret_cast<float*>(static_cast<char*>(workspace) + lay.lse_tok);
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, sa::tw_tile_tokens(), st); }));
+  return tw_forward(a, lay, sketch, lse_tok, st);
+}
+
+sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
+                                  const void* Q, int H, int P, int d, float scale, sa_dtype dt, const float* sketch,
+                                  const float* lse_tok, const float* dsketch, void* dK, void* dV, float* dQ,
+                                  void* workspace, size_t ws_bytes, void* stream) {
+  if (!dsketch || !dQ || (N > 0 && (!dK || !dV))) return SA_ERR_INVALID_ARG;
+  TwLayout lay;
+  SA_TRY(tw_check(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, true, &lay));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* base = static_cast<char*>(workspace);
+  sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, lay.base);
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, sa::tw_tile_tokens(), st); }));
+  if (!sketch || !lse_tok) {  // recompute both from the inputs
+    float* O = reinterpret_cast<float*>(base + lay.sketch);
+    float* l = reinterpret_cast<float*>(base + lay.lse_tok);
+    SA_TRY(tw_forward(a, lay, O, l, st));
+    sketch = O;
+    lse_tok = l;
+  }
+  float* D = reinterpret_cast<float*>(base + lay.dcoef);
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tw_dcoef(a, sketch, dsketch, D, st); }));
+  SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
+                [&] { return sa::launch_tw_bwd_tokens(a, dsketch, lse_tok, D, dK, dV, st); }));
+  SA_TRY(launch(SA_KERNEL_BWD_DQ, st, [&] { return sa::launch_tw_bwd_dq(a, lay.W, dsketch, lse_tok, D, st); }));
+  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, lay.W, dQ, st); });
 }
 
 sa_status sa_get_device_error(const void* workspace, void* stream) {

@@ -50,4 +50,15 @@ cudaError_t launch_simt_bwd_tokens(const Args& a, const float* dsk, const float*
 cudaError_t launch_simt_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
                                cudaStream_t st);
 
+// token-wise normalisation (sa_tokenwise.cu)
+int tw_tile_tokens();
+cudaError_t launch_tw_fwd(const Args& a, int W, float* sketch, float* lse_tok, float2* stat_part, cudaStream_t st);
+cudaError_t launch_tw_finalize(const Args& a, int W, const float2* stat_part, float* sketch, float* lse_tok,
+                               cudaStream_t st);
+cudaError_t launch_tw_dcoef(const Args& a, const float* O, const float* G, float* D, cudaStream_t st);
+cudaError_t launch_tw_bwd_tokens(const Args& a, const float* dsk, const float* lse_tok, const float* D, void* dK,
+                                 void* dV, cudaStream_t st);
+cudaError_t launch_tw_bwd_dq(const Args& a, int W, const float* dsk, const float* lse_tok, const float* D,
+                             cudaStream_t st);
+
 }  // namespace sa

@@ -96,3 +96,27 @@ def test_plan_host_rejects_bad_offsets(lib):
         binding.sa_plan_host(np.array([0, 5, 3], np.int32), 1, 128, 4)
     with pytest.raises(binding.SketchError):
         binding.sa_plan_host(np.array([1, 5], np.int32), 1, 128, 4)
+
+
+def test_tokenwise_host_checks(lib):
+    vp = ctypes.c_void_p
+
+    def fwd(**kw):
+        a = dict(K=256, V=512, cu=768, B=2, N=100, Q=1024, H=2, P=64, d=64, scale=0.125, dt=1, sketch=2048,
+                 ws=4096, wsb=1 << 30)
+        a.update(kw)
+        return lib.sa_sketch_fwd_tokenwise(vp(a["K"]), vp(a["V"]), vp(a["cu"]), a["B"], a["N"], vp(a["Q"]), a["H"],
+                                           a["P"], a["d"], a["scale"], a["dt"], vp(a["sketch"]) if a["sketch"] else None,
+                                           None, vp(a["ws"]), a["wsb"], None)
+
+    assert fwd(sketch=0) == 1
+    assert fwd(ws=4096 + 8) == 1
+    assert fwd(P=4096) == 2
+    assert fwd(wsb=16) == 3
+    bwd = lib.sa_sketch_bwd_tokenwise(vp(256), vp(512), vp(768), 2, 100, vp(1024), 2, 64, 64, 0.125, 1, None, None,
+                                      None, vp(2048), vp(2304), vp(2560), vp(4096), 1 << 30, None)
+    assert bwd == 1  # NULL dsketch
+    a = binding.load().sa_workspace_size_tokenwise(4, 1000, 2, 256, 64, 1, 0)
+    b = binding.load().sa_workspace_size_tokenwise(4, 1000, 2, 256, 64, 1, 1)
+    assert a > 0 and b > a and a % 256 == 0 and b % 256 == 0
+    assert binding.load().sa_workspace_size_tokenwise(1, 10, 1, 4096, 64, 1, 0) == 0
