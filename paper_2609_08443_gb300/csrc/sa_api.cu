@@ -413,29 +413,37 @@ sa_status sa_sketch_bwd_x(const void* X, const int32_t* cu_seqlens, int B, int64
 // ------------------------------ token-wise normalisation (Sec. 5.1, App. C)
 namespace {
 
-// Workspace of the token-wise entry points (CUDA-core kernels, 32-token tiles):
-// header | tile prefix | cut-segment pieces [W][2][P][d] | dQ pieces [W][H][P][d]
-// (bwd) | piece statistics float2 [W][2][P] | lse_tok [B][H][P] | D [B][H][P] (bwd)
-// | sketch recomputed by the backward [B][H][P][d] (bwd).
+// Workspace of the token-wise entry points: header | tile prefix | cut-segment
+// pieces [Wf][2][P][d] | dQ pieces [Wb][H][P][d] (bwd) | piece statistics
+// float2 [Wf][2][P] | lse_tok [B][H][P] | D [B][H][P] (bwd) | sketch recomputed
+// by the backward [B][H][P][d] (bwd).  The forward runs on the tensor cores
+// (128-token tiles, Wf workers) where tc_tw_fwd_supported, else on CUDA cores
+// (32-token tiles); the backward always on CUDA cores (32-token tiles, Wb).
 struct TwLayout {
   sa::WsLayout base;
   size_t stat_part, lse_tok, dcoef, sketch, total;
-  int W;
+  bool tc_fwd;
+  int Tf, Wf, Tb, Wb;
 };
 
-TwLayout tw_layout(int B, int H, int P, int d, bool bwd) {
+TwLayout tw_layout(int B, int H, int P, int d, sa_dtype dt, float scale, bool bwd) {
   TwLayout t{};
-  t.W = sa::simt_workers(device_sms() > 0 ? device_sms() : 1, P);
+  const int sms = device_sms() > 0 ? device_sms() : 1;
+  t.tc_fwd = sa::tc_tw_fwd_supported(P, d, dt, scale);
+  t.Tf = t.tc_fwd ? sa::tc_tile_tokens() : sa::tw_tile_tokens();
+  t.Wf = t.tc_fwd ? sa::tc_tw_fwd_workers(sms, P) : sa::simt_workers(sms, P);
+  t.Tb = sa::tw_tile_tokens();
+  t.Wb = sa::simt_workers(sms, P);
   sa::WsLayout& L = t.base;
   size_t off = sizeof(sa::WsHeader);
   L.tile_prefix = off;
   off = sa::align256(off + sizeof(int64_t) * size_t(B + 1));
   L.partial = off;
-  off = sa::align256(off + sizeof(float) * size_t(t.W) * 2 * P * d);
+  off = sa::align256(off + sizeof(float) * size_t(t.Wf) * 2 * P * d);
   L.dq_partial = off;
-  if (bwd) off = sa::align256(off + sizeof(float) * size_t(t.W) * H * P * d);
+  if (bwd) off = sa::align256(off + sizeof(float) * size_t(t.Wb) * H * P * d);
   t.stat_part = off;
-  off = sa::align256(off + sizeof(float2) * size_t(t.W) * 2 * P);
+  off = sa::align256(off + sizeof(float2) * size_t(t.Wf) * 2 * P);
   t.lse_tok = off;
   off = sa::align256(off + sizeof(float) * size_t(B) * H * P);
   t.dcoef = off;
@@ -453,22 +461,29 @@ TwLayout tw_layout(int B, int H, int P, int d, bool bwd) {
 sa_status tw_check(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q, int H, int P,
                    int d, float scale, sa_dtype dt, const void* ws, size_t ws_bytes, bool bwd, TwLayout* lay) {
   SA_TRY(check_args(K, V, cu, B, N, Q, H, P, d, scale, dt, ws));
-  *lay = tw_layout(B, H, P, d, bwd);
+  *lay = tw_layout(B, H, P, d, dt, scale, bwd);
   return ws_bytes < lay->total ? SA_ERR_WORKSPACE : SA_OK;
 }
 
-// Plan, online-softmax sweep, merge of cut segments: sketch and lse_tok.
+// Plan for the forward's tiles, online-softmax sweep, merge of cut segments:
+// sketch and lse_tok.
 sa_status tw_forward(const sa::Args& a, const TwLayout& lay, float* sketch, float* lse_tok, cudaStream_t st) {
   float2* stat = reinterpret_cast<float2*>(static_cast<char*>(a.ws) + lay.stat_part);
-  SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_tw_fwd(a, lay.W, sketch, lse_tok, stat, st); }));
-  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tw_finalize(a, lay.W, stat, sketch, lse_tok, st); });
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, lay.Tf, st); }));
+  if (lay.tc_fwd) {
+    SA_TRY(launch(SA_KERNEL_FWD_MAIN, st,
+                  [&] { return sa::launch_tc_tw_fwd(a, lay.Wf, sketch, lse_tok, stat, st); }));
+  } else {
+    SA_TRY(launch(SA_KERNEL_FWD_MAIN, st, [&] { return sa::launch_tw_fwd(a, lay.Wf, sketch, lse_tok, stat, st); }));
+  }
+  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tw_finalize(a, lay.Wf, stat, sketch, lse_tok, st); });
 }
 
 }  // namespace
 
 size_t sa_workspace_size_tokenwise(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd) {
   if (!shape_ok(B, N, H, P, d, dt)) return 0;
-  return tw_layout(B, H, P, d, bwd != 0).total;
+  return tw_layout(B, H, P, d, dt, 1.f, bwd != 0).total;
 }
 
 sa_status sa_sketch_fwd_tokenwise(const void* K, const void* V, const int32_t* cu_seqlens, int B, int64_t N,
@@ -480,7 +495,6 @@ sa_status sa_sketch_fwd_tokenwise(const void* K, const void* V, const int32_t* c
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, lay.base);
   if (!lse_tok) lse_tok = reinterpret_cast<float*>(static_cast<char*>(workspace) + lay.lse_tok);
-  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, sa::tw_tile_tokens(), st); }));
   return tw_forward(a, lay, sketch, lse_tok, st);
 }
 
@@ -494,7 +508,6 @@ sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* c
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   char* base = static_cast<char*>(workspace);
   sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, lay.base);
-  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, sa::tw_tile_tokens(), st); }));
   if (!sketch || !lse_tok) {  // recompute both from the inputs
     float* O = reinterpret_cast<float*>(base + lay.sketch);
     float* l = reinterpret_cast<float*>(base + lay.lse_tok);
@@ -502,12 +515,13 @@ sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* c
     sketch = O;
     lse_tok = l;
   }
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, lay.Tb, st); }));
   float* D = reinterpret_cast<float*>(base + lay.dcoef);
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tw_dcoef(a, sketch, dsketch, D, st); }));
   SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
                 [&] { return sa::launch_tw_bwd_tokens(a, dsketch, lse_tok, D, dK, dV, st); }));
-  SA_TRY(launch(SA_KERNEL_BWD_DQ, st, [&] { return sa::launch_tw_bwd_dq(a, lay.W, dsketch, lse_tok, D, st); }));
-  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, lay.W, dQ, st); });
+  SA_TRY(launch(SA_KERNEL_BWD_DQ, st, [&] { return sa::launch_tw_bwd_dq(a, lay.Wb, dsketch, lse_tok, D, st); }));
+  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, lay.Wb, dQ, st); });
 }
 
 sa_status sa_get_device_error(const void* workspace, void* stream) {

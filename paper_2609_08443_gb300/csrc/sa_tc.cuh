@@ -26,6 +26,12 @@ cudaError_t launch_tc_bwd_tok(const Args& a, int W, const float* dsk, __nv_bfloa
 cudaError_t launch_tc_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
                              cudaStream_t st);
 int tc_bwd_dq_workers(int num_sms, int P);
+// token-wise normalisation (Sec. 5.1): tensor-core forward
+bool tc_tw_fwd_supported(int P, int d, sa_dtype dt, float scale);
+int tc_tw_fwd_workers(int num_sms, int P);
+const char* tc_tw_fwd_name(int P, int d);
+cudaError_t launch_tc_tw_fwd(const Args& a, int W, float* sketch, float* lse_tok, float2* stat_part,
+                             cudaStream_t st);
 cudaError_t launch_tc_g_bf16(const Args& a, const float* dsk, __nv_bfloat16* gbf, cudaStream_t st);
 
 }  // namespace sa
