@@ -161,7 +161,9 @@ sa_status sa_sketch_fwd_tokenwise(const void* K, const void* V, const int32_t* c
  *     dV_i = sum_j A[j,i] G_j,    dS[j,i] = A[j,i] (G_j . v_i - D_j),
  *     dK_i = scale sum_j dS[j,i] Q_j,    dQ[h] = scale sum_b sum_i dS[:,i] K_b[i,h].
  * `sketch` and `lse_tok` are the forward's outputs; when either is NULL both are
- * recomputed.  dK, dV have type `dt`, dQ is fp32; all fully overwritten. */
+ * recomputed.  sketch, lse_tok and dsketch must be 16-byte aligned.  dK, dV have
+ * type `dt`, dQ is fp32; all fully overwritten.  Tensor cores serve bf16 with
+ * d = 128 and P in {256, 512, 1024, 2048}; other shapes run on CUDA cores. */
 sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* cu_seqlens, int B,
                                   int64_t N, const void* Q, int H, int P, int d, float scale,
                                   sa_dtype dt, const float* sketch, const float* lse_tok,

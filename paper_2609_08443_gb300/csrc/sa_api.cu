@@ -414,26 +414,30 @@ sa_status sa_sketch_bwd_x(const void* X, const int32_t* cu_seqlens, int B, int64
 namespace {
 
 // Workspace of the token-wise entry points: header | tile prefix | cut-segment
-// pieces [Wf][2][P][d] | dQ pieces [Wb][H][P][d] (bwd) | piece statistics
+// pieces [Wf][2][P][d] | dQ pieces [Wq][H][P][d] (bwd) | piece statistics
 // float2 [Wf][2][P] | lse_tok [B][H][P] | D [B][H][P] (bwd) | sketch recomputed
-// by the backward [B][H][P][d] (bwd).  The forward runs on the tensor cores
-// (128-token tiles, Wf workers) where tc_tw_fwd_supported, else on CUDA cores
-// (32-token tiles); the backward always on CUDA cores (32-token tiles, Wb).
+// by the backward [B][H][P][d] (bwd) | bf16 copy of dsketch (bwd, tensor cores).
+// The forward runs on the tensor cores (128-token tiles, Wf workers) where
+// tc_tw_fwd_supported, else on CUDA cores (32-token tiles); the backward on the
+// tensor cores (token side with Wb workers, dQ with Wq) where
+// tc_tw_bwd_supported, else on CUDA cores (Wb = Wq workers).
 struct TwLayout {
   sa::WsLayout base;
-  size_t stat_part, lse_tok, dcoef, sketch, total;
-  bool tc_fwd;
-  int Tf, Wf, Tb, Wb;
+  size_t stat_part, lse_tok, dcoef, sketch, gbf, total;
+  bool tc_fwd, tc_bwd;
+  int Tf, Wf, Tb, Wb, Wq;
 };
 
 TwLayout tw_layout(int B, int H, int P, int d, sa_dtype dt, float scale, bool bwd) {
   TwLayout t{};
   const int sms = device_sms() > 0 ? device_sms() : 1;
   t.tc_fwd = sa::tc_tw_fwd_supported(P, d, dt, scale);
+  t.tc_bwd = sa::tc_tw_bwd_supported(P, d, dt);
   t.Tf = t.tc_fwd ? sa::tc_tile_tokens() : sa::tw_tile_tokens();
   t.Wf = t.tc_fwd ? sa::tc_tw_fwd_workers(sms, P) : sa::simt_workers(sms, P);
-  t.Tb = sa::tw_tile_tokens();
-  t.Wb = sa::simt_workers(sms, P);
+  t.Tb = t.tc_bwd ? sa::tc_tile_tokens() : sa::tw_tile_tokens();
+  t.Wb = t.tc_bwd ? sa::tc_bwd_workers(sms, P, d) : sa::simt_workers(sms, P);
+  t.Wq = t.tc_bwd ? sa::tc_bwd_dq_workers(sms, P) : t.Wb;
   sa::WsLayout& L = t.base;
   size_t off = sizeof(sa::WsHeader);
   L.tile_prefix = off;
@@ -441,17 +445,18 @@ TwLayout tw_layout(int B, int H, int P, int d, sa_dtype dt, float scale, bool bw
   L.partial = off;
   off = sa::align256(off + sizeof(float) * size_t(t.Wf) * 2 * P * d);
   L.dq_partial = off;
-  if (bwd) off = sa::align256(off + sizeof(float) * size_t(t.Wb) * H * P * d);
+  if (bwd) off = sa::align256(off + sizeof(float) * size_t(t.Wq) * H * P * d);
   t.stat_part = off;
   off = sa::align256(off + sizeof(float2) * size_t(t.Wf) * 2 * P);
   t.lse_tok = off;
   off = sa::align256(off + sizeof(float) * size_t(B) * H * P);
-  t.dcoef = off;
-  t.sketch = off;
+  t.dcoef = t.sketch = t.gbf = off;
   if (bwd) {
     off = sa::align256(off + sizeof(float) * size_t(B) * H * P);
     t.sketch = off;
     off = sa::align256(off + sizeof(float) * size_t(B) * H * P * d);
+    t.gbf = off;
+    if (t.tc_bwd) off = sa::align256(off + 2 * size_t(B) * H * P * d);
   }
   L.lse = L.dcoef = L.gbf = L.lse_part = off;  // unused on this path
   L.total = t.total = off;
@@ -503,6 +508,8 @@ sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* c
                                   const float* lse_tok, const float* dsketch, void* dK, void* dV, float* dQ,
                                   void* workspace, size_t ws_bytes, void* stream) {
   if (!dsketch || !dQ || (N > 0 && (!dK || !dV))) return SA_ERR_INVALID_ARG;
+  if ((sketch && !aligned16(sketch)) || (lse_tok && !aligned16(lse_tok)) || !aligned16(dsketch))
+    return SA_ERR_INVALID_ARG;
   TwLayout lay;
   SA_TRY(tw_check(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, true, &lay));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -517,11 +524,21 @@ sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* c
   }
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, lay.Tb, st); }));
   float* D = reinterpret_cast<float*>(base + lay.dcoef);
-  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tw_dcoef(a, sketch, dsketch, D, st); }));
-  SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
-                [&] { return sa::launch_tw_bwd_tokens(a, dsketch, lse_tok, D, dK, dV, st); }));
-  SA_TRY(launch(SA_KERNEL_BWD_DQ, st, [&] { return sa::launch_tw_bwd_dq(a, lay.Wb, dsketch, lse_tok, D, st); }));
-  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, lay.Wb, dQ, st); });
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tw_dcoef(a, sketch, dsketch, lay.tc_bwd, D, st); }));
+  if (lay.tc_bwd) {
+    __nv_bfloat16* gbf = reinterpret_cast<__nv_bfloat16*>(base + lay.gbf);
+    SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_tc_g_bf16(a, dsketch, gbf, st); }));
+    SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
+                  [&] { return sa::launch_tc_tw_bwd_tok(a, lay.Wb, gbf, lse_tok, D, dK, dV, st); }));
+    SA_TRY(launch(SA_KERNEL_BWD_DQ, st,
+                  [&] { return sa::launch_tc_tw_bwd_dq(a, lay.Wq, dsketch, lse_tok, D, st); }));
+  } else {
+    SA_TRY(launch(SA_KERNEL_BWD_MAIN, st,
+                  [&] { return sa::launch_tw_bwd_tokens(a, dsketch, lse_tok, D, dK, dV, st); }));
+    SA_TRY(launch(SA_KERNEL_BWD_DQ, st,
+                  [&] { return sa::launch_tw_bwd_dq(a, lay.Wb, dsketch, lse_tok, D, st); }));
+  }
+  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, lay.Wq, dQ, st); });
 }
 
 sa_status sa_get_device_error(const void* workspace, void* stream) {

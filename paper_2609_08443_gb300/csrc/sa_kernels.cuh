@@ -55,7 +55,8 @@ int tw_tile_tokens();
 cudaError_t launch_tw_fwd(const Args& a, int W, float* sketch, float* lse_tok, float2* stat_part, cudaStream_t st);
 cudaError_t launch_tw_finalize(const Args& a, int W, const float2* stat_part, float* sketch, float* lse_tok,
                                cudaStream_t st);
-cudaError_t launch_tw_dcoef(const Args& a, const float* O, const float* G, float* D, cudaStream_t st);
+cudaError_t launch_tw_dcoef(const Args& a, const float* O, const float* G, bool round_g, float* D,
+                            cudaStream_t st);
 cudaError_t launch_tw_bwd_tokens(const Args& a, const float* dsk, const float* lse_tok, const float* D, void* dK,
                                  void* dV, cudaStream_t st);
 cudaError_t launch_tw_bwd_dq(const Args& a, int W, const float* dsk, const float* lse_tok, const float* D,

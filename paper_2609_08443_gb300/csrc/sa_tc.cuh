@@ -32,6 +32,11 @@ int tc_tw_fwd_workers(int num_sms, int P);
 const char* tc_tw_fwd_name(int P, int d);
 cudaError_t launch_tc_tw_fwd(const Args& a, int W, float* sketch, float* lse_tok, float2* stat_part,
                              cudaStream_t st);
+bool tc_tw_bwd_supported(int P, int d, sa_dtype dt);
+cudaError_t launch_tc_tw_bwd_tok(const Args& a, int W, const __nv_bfloat16* gbf, const float* lse_tok,
+                                 const float* Dtw, void* dK, void* dV, cudaStream_t st);
+cudaError_t launch_tc_tw_bwd_dq(const Args& a, int W, const float* dsk, const float* lse_tok, const float* Dtw,
+                                cudaStream_t st);
 cudaError_t launch_tc_g_bf16(const Args& a, const float* dsk, __nv_bfloat16* gbf, cudaStream_t st);
 
 }  // namespace sa

@@ -637,13 +637,16 @@ struct TokCfg {
 __device__ __forceinline__ int tok_kv_pair(int) { return 0; }
 __device__ __forceinline__ int tok_qg_pair(int, int c) { return 1 + (c & 1); }
 
-template <int D, int P>
-__global__ void __launch_bounds__(kThreads, 1)
-    tc_bwd_tok_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                      const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmG,
-                      const __grid_constant__ CUtensorMap tmDK, const __grid_constant__ CUtensorMap tmDV, Args a,
-                      const float* __restrict__ lse, float* __restrict__ Dco, __nv_bfloat16* __restrict__ dK,
-                      __nv_bfloat16* __restrict__ dV) {
+// TW = false: prototype-wise weights (Sec. 3.1), lse and Dco per token [N][H]
+// (Dco written here).  TW = true: token-wise weights (Sec. 5.1), lse and Dco
+// per prototype [B][H][P] (both read), so dS = A o (dA - D_j) goes to shared
+// memory in place of E and dK = scale dS Q needs no qbar.
+template <int D, int P, bool TW>
+__device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUtensorMap& tmV, const CUtensorMap& tmQ,
+                                             const CUtensorMap& tmG, const CUtensorMap& tmDK,
+                                             const CUtensorMap& tmDV, const Args& a, const float* __restrict__ lse,
+                                             float* __restrict__ Dco, __nv_bfloat16* __restrict__ dK,
+                                             __nv_bfloat16* __restrict__ dV) {
   using C = TokCfg<D, P>;
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -755,7 +758,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // descriptors are built once per operand and stepped by constant offsets,
       // so the issue loop carries no address arithmetic.
       constexpr uint32_t idS = idesc_bf16(128, C::NC, 0, 0);    // [tok x chunk], K = d
-      constexpr uint32_t idGQ = idesc_bf16(128, 2 * D, 0, 1);   // [tok x (d | d)], K = chunk prototypes
+      constexpr uint32_t idGQ = idesc_bf16(128, TW ? D : 2 * D, 0, 1);  // [tok x (d | d)] (TW: d), K = chunk
       constexpr uint32_t idU = idesc_bf16(128, D, 0, 1);        // [tok x d], K = chunk prototypes
       bool ok = true;
       int uses[C::NSLOT] = {0, 0, 0, 0, 0, 0};
@@ -887,21 +890,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++epi;
         return r;
       };
-      float lse_cur = row < cur.n ? lse[(cur.tok0 + row) * a.H + cur.h] : 0.f;
+      float lse_cur = (!TW && row < cur.n) ? lse[(cur.tok0 + row) * a.H + cur.h] : 0.f;
       for (int li = 0; li < ntiles && ok; ++li) {
         const bool valid = row < cur.n;
         const int64_t tok = cur.tok0 + row;
         const float L2 = lse_cur * 1.4426950408889634f;
-        {
+        if (!TW) {
           int64_t t0n;
           int nn, hn;
           cur.peek_next(t0n, nn, hn);
           lse_cur = row < nn ? lse[(t0n + row) * a.H + hn] : 0.f;
         }
+        // token-wise: this segment's per-prototype lse and D_j (the same for
+        // every thread: broadcast loads)
+        const int64_t seg_row = (int64_t(cur.b) * a.H + cur.h) * a.P;
         float Dp = 0.f;
         for (int c = 0; c < C::NCH && ok; ++c, ++g) {
           uint32_t apk[C::HALF / 2];
           float v[32];
+          const int j0 = c * C::NC + sw * C::HALF;  // first prototype of this warpgroup's columns
           ok = wwait(s_full, g & 1, 0xA01);
           if (!ok) break;
           tc_fence_after();
@@ -909,11 +916,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int cc = 0; cc < C::HALF / 32; ++cc) {
             tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * cc, v);
             tmem_ld_wait();
+            if (TW) {
+              const float4* l4 = reinterpret_cast<const float4*>(lse + seg_row + j0 + 32 * cc);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              const float x0 = valid ? ex2(fmaf(v[2 * j], c2, -L2)) : 0.f;
-              const float x1 = valid ? ex2(fmaf(v[2 * j + 1], c2, -L2)) : 0.f;
-              apk[16 * cc + j] = pack_bf16(x0, x1);
+              for (int j4 = 0; j4 < 8; ++j4) {
+                const float4 l = __ldg(l4 + j4);
+                const float x0 = valid ? ex2(fmaf(v[4 * j4 + 0], c2, -l.x * 1.4426950408889634f)) : 0.f;
+                const float x1 = valid ? ex2(fmaf(v[4 * j4 + 1], c2, -l.y * 1.4426950408889634f)) : 0.f;
+                const float x2 = valid ? ex2(fmaf(v[4 * j4 + 2], c2, -l.z * 1.4426950408889634f)) : 0.f;
+                const float x3 = valid ? ex2(fmaf(v[4 * j4 + 3], c2, -l.w * 1.4426950408889634f)) : 0.f;
+                apk[16 * cc + 2 * j4] = pack_bf16(x0, x1);
+                apk[16 * cc + 2 * j4 + 1] = pack_bf16(x2, x3);
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const float x0 = valid ? ex2(fmaf(v[2 * j], c2, -L2)) : 0.f;
+                const float x1 = valid ? ex2(fmaf(v[2 * j + 1], c2, -L2)) : 0.f;
+                apk[16 * cc + j] = pack_bf16(x0, x1);
+              }
             }
           }
           tc_fence_before();
@@ -927,7 +948,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(a_full);
-          // E = A o dA
+          // E = A o dA (token-wise: dS = A o (dA - D_j))
           ok = wwait(da_full, g & 1, 0xA03);
           if (!ok) break;
           tc_fence_after();
@@ -936,12 +957,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int cc = 0; cc < C::HALF / 32; ++cc) {
             tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * cc, v);
             tmem_ld_wait();
+            if (TW) {
+              const float4* d4 = reinterpret_cast<const float4*>(Dco + seg_row + j0 + 32 * cc);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              const uint32_t w = apk[16 * cc + j];
-              const float e0 = bf16lo(w) * v[2 * j], e1 = bf16hi(w) * v[2 * j + 1];
-              Dp += e0 + e1;
-              epk[16 * cc + j] = pack_bf16(e0, e1);
+              for (int j4 = 0; j4 < 8; ++j4) {
+                const float4 dd = __ldg(d4 + j4);
+                const uint32_t w0 = apk[16 * cc + 2 * j4], w1 = apk[16 * cc + 2 * j4 + 1];
+                epk[16 * cc + 2 * j4] = pack_bf16(bf16lo(w0) * (v[4 * j4 + 0] - dd.x),
+                                                  bf16hi(w0) * (v[4 * j4 + 1] - dd.y));
+                epk[16 * cc + 2 * j4 + 1] = pack_bf16(bf16lo(w1) * (v[4 * j4 + 2] - dd.z),
+                                                      bf16hi(w1) * (v[4 * j4 + 3] - dd.w));
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const uint32_t w = apk[16 * cc + j];
+                const float e0 = bf16lo(w) * v[2 * j], e1 = bf16hi(w) * v[2 * j + 1];
+                Dp += e0 + e1;
+                epk[16 * cc + j] = pack_bf16(e0, e1);
+              }
             }
           }
           tc_fence_before();
@@ -955,20 +989,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) mbar_arrive(e_full);
         }
         if (!ok) break;
-        // D_i = (half from warpgroup 0) + (half from warpgroup 1), same order in both
-        if (li > 0) {
-          ok = wwait(st_used, (li - 1) & 1, 0xA05);
+        // D_i = (half from warpgroup 0) + (half from warpgroup 1), same order in
+        // both; token-wise: u already is sum_j dS[j,i] Q_j, so D_i = 0 below
+        float Dv = 0.f;
+        if (!TW) {
+          if (li > 0) {
+            ok = wwait(st_used, (li - 1) & 1, 0xA05);
+            if (!ok) break;
+          }
+          stats[sw * T + row] = Dp;
+          __syncwarp();
+          if (lane == 0) mbar_arrive(st_ready);
+          ok = wwait(st_ready, li & 1, 0xA06);
           if (!ok) break;
+          Dv = stats[row] + stats[T + row];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(st_used);
+          if (sw == 0 && valid) Dco[tok * a.H + cur.h] = Dv;
         }
-        stats[sw * T + row] = Dp;
-        __syncwarp();
-        if (lane == 0) mbar_arrive(st_ready);
-        ok = wwait(st_ready, li & 1, 0xA06);
-        if (!ok) break;
-        const float Dv = stats[row] + stats[T + row];
-        __syncwarp();
-        if (lane == 0) mbar_arrive(st_used);
-        if (sw == 0 && valid) Dco[tok * a.H + cur.h] = Dv;
         // epilogue: dV and dK = scale (u - D qbar); this warpgroup owns columns [sw*D/2, +D/2)
         ok = wwait(acc_full, li & 1, 0xA07);
         if (!ok) break;
@@ -999,10 +1037,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int cc = 0; cc < D / 2; cc += 32) {
             tmem_ld32(tmem + lane_off + C::U_COL + sw * (D / 2) + cc, uu);
-            tmem_ld32(tmem + lane_off + C::QB_COL + sw * (D / 2) + cc, qb);
+            if (!TW) tmem_ld32(tmem + lane_off + C::QB_COL + sw * (D / 2) + cc, qb);
             tmem_ld_wait();
 #pragma unroll
-            for (int j = 0; j < 32; ++j) uu[j] = a.scale * fmaf(-Dv, qb[j], uu[j]);
+            for (int j = 0; j < 32; ++j) uu[j] = TW ? a.scale * uu[j] : a.scale * fmaf(-Dv, qb[j], uu[j]);
             put_half(uu, cc);
           }
           ok = stage_and_store(&tmDK, cur);
@@ -1015,7 +1053,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int cc = 0; cc < D / 2; cc += 32) {
             tmem_ld32(tmem + lane_off + C::U_COL + sw * (D / 2) + cc, uu);
-            tmem_ld32(tmem + lane_off + C::QB_COL + sw * (D / 2) + cc, qb);
+            if (!TW) tmem_ld32(tmem + lane_off + C::QB_COL + sw * (D / 2) + cc, qb);
             tmem_ld_wait();
             if (valid) {
               uint4* o = reinterpret_cast<uint4*>(dkr + cc);
@@ -1023,7 +1061,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               for (int k = 0; k < 4; ++k) {
                 float x[8];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) x[j] = a.scale * fmaf(-Dv, qb[8 * k + j], uu[8 * k + j]);
+                for (int j = 0; j < 8; ++j)
+                  x[j] = TW ? a.scale * uu[8 * k + j] : a.scale * fmaf(-Dv, qb[8 * k + j], uu[8 * k + j]);
                 o[k] = make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]),
                                   pack_bf16(x[6], x[7]));
               }
@@ -1045,6 +1084,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+template <int D, int P>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_bwd_tok_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                      const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmG,
+                      const __grid_constant__ CUtensorMap tmDK, const __grid_constant__ CUtensorMap tmDV, Args a,
+                      const float* __restrict__ lse, float* __restrict__ Dco, __nv_bfloat16* __restrict__ dK,
+                      __nv_bfloat16* __restrict__ dV) {
+  bwd_tok_body<D, P, false>(tmK, tmV, tmQ, tmG, tmDK, tmDV, a, lse, Dco, dK, dV);
+}
+
+template <int D, int P>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_tw_bwd_tok_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                         const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmG,
+                         const __grid_constant__ CUtensorMap tmDK, const __grid_constant__ CUtensorMap tmDV, Args a,
+                         const float* __restrict__ lse_tok, float* __restrict__ Dtw, __nv_bfloat16* __restrict__ dK,
+                         __nv_bfloat16* __restrict__ dV) {
+  bwd_tok_body<D, P, true>(tmK, tmV, tmQ, tmG, tmDK, tmDV, a, lse_tok, Dtw, dK, dV);
+}
+
 // dsketch fp32 -> bf16 copy in the workspace, the layout TMA streams ([B*H][P][D])
 __global__ void to_bf16_kernel(const float* __restrict__ src, __nv_bfloat16* __restrict__ dst, int64_t n8,
                                const void* ws) {
@@ -1057,7 +1116,7 @@ __global__ void to_bf16_kernel(const float* __restrict__ src, __nv_bfloat16* __r
   }
 }
 
-template <int D, int P>
+template <int D, int P, bool TW = false>
 static cudaError_t launch_tok_t(const Args& a, int W, const __nv_bfloat16* gbf, const float* lse, float* Dco,
                                 void* dK, void* dV, cudaStream_t st) {
   using C = TokCfg<D, P>;
@@ -1066,7 +1125,7 @@ static cudaError_t launch_tok_t(const Args& a, int W, const __nv_bfloat16* gbf, 
       !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, C::NC) || !make_q_map(&tg, gbf, a.B * a.H, a.P, D, C::NC) ||
       !make_kv_map(&tdk, dK, a.N, a.H, D) || !make_kv_map(&tdv, dV, a.N, a.H, D))
     return cudaErrorInvalidValue;
-  auto fn = &tc_bwd_tok_kernel<D, P>;
+  auto fn = TW ? &tc_tw_bwd_tok_kernel<D, P> : &tc_bwd_tok_kernel<D, P>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   fn<<<W, kThreads, C::SMEM, st>>>(tk, tv, tq, tg, tdk, tdv, a, lse, Dco, static_cast<__nv_bfloat16*>(dK),
@@ -1144,11 +1203,14 @@ struct QCfg {
 // the UMMA issuer follows the tile sequence without walking it.
 enum : uint32_t { kNewHead = 1u, kHeadLast = 2u, kSegFirst = 4u, kSegLast = 8u };
 
-template <int D, int PS>
-__global__ void __launch_bounds__(kThreads, 1)
-    tc_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                     const __grid_constant__ CUtensorMap tmQ, Args a, const float* __restrict__ dsk,
-                     const float* __restrict__ lse, const float* __restrict__ Dco) {
+// TW = false: prototype-wise weights, lse and D per token (column values
+// staged by warps 2-3).  TW = true: token-wise weights (Sec. 5.1), lse and D
+// per prototype [B][H][P]: per-row (per-thread) values, and columns past the
+// tile's tokens are masked here.
+template <int D, int PS, bool TW>
+__device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtensorMap& tmV, const CUtensorMap& tmQ,
+                                            const Args& a, const float* __restrict__ dsk,
+                                            const float* __restrict__ lse, const float* __restrict__ Dco) {
   using C = QCfg<D, PS>;
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1364,18 +1426,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) mbar_arrive(g_full);
           ++gc;
         }
-        const int buf = li & 1;
-        if (li >= 2) ok = hw(col_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xE02);
-        if (!ok) break;
-        float* cl = cols + buf * 2 * T;
-        for (int t = t64; t < T; t += 64) {
-          const bool v = t < cur.n;
-          const int64_t idx = (cur.tok0 + t) * a.H + cur.h;
-          cl[t] = v ? lse[idx] * 1.4426950408889634f : INFINITY;  // exp2(x - inf) = 0 for padding
-          cl[T + t] = v ? Dco[idx] : 0.f;
+        if (!TW) {
+          const int buf = li & 1;
+          if (li >= 2) ok = hw(col_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xE02);
+          if (!ok) break;
+          float* cl = cols + buf * 2 * T;
+          for (int t = t64; t < T; t += 64) {
+            const bool v = t < cur.n;
+            const int64_t idx = (cur.tok0 + t) * a.H + cur.h;
+            cl[t] = v ? lse[idx] * 1.4426950408889634f : INFINITY;  // exp2(x - inf) = 0 for padding
+            cl[T + t] = v ? Dco[idx] : 0.f;
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(col_full0 + 8 * buf);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(col_full0 + 8 * buf);
         cur.next();
       }
     } else if (warp >= kSoftWarp0) {
@@ -1391,7 +1455,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       int hp = 0;
       for (int li = 0; li < ntiles && ok; ++li) {
         const int buf = li & 1;
-        ok = wwait(col_full0 + 8 * buf, (li >> 1) & 1, 0xF01);
+        float l2r = 0.f, dr = 0.f;  // token-wise: this row's lse (log2 units) and D
+        if (TW) {
+          const int64_t r = (int64_t(cur.b) * a.H + cur.h) * a.P + p0 + 32 * q + lane;
+          l2r = lse[r] * 1.4426950408889634f;
+          dr = Dco[r];
+        } else {
+          ok = wwait(col_full0 + 8 * buf, (li >> 1) & 1, 0xF01);
+        }
         if (ok) ok = wwait(sda_full, li & 1, 0xF02);
         // this tile's dS buffer was last read by dQ(i-2)
         if (ok && li > 1) ok = wwait(ds_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xF04);
@@ -1407,10 +1478,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(sda_free);  // the next tile's S and dA may now be written
+        if (TW) {
+          // per-row shift and D; columns past the tile's tokens weigh zero
+#pragma unroll
+          for (int c = 0; c < 2; ++c) {
+            const int col = 64 * sw + 32 * c;
+            uint32_t pk[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const int jj = 32 * c + 2 * j;
+              const float a0 = col + 2 * j < cur.n ? ex2(fmaf(sv[jj], c2, -l2r)) : 0.f;
+              const float a1 = col + 2 * j + 1 < cur.n ? ex2(fmaf(sv[jj + 1], c2, -l2r)) : 0.f;
+              pk[j] = pack_bf16(a0 * (dv[jj] - dr), a1 * (dv[jj + 1] - dr));
+            }
+            tmem_st16(tmem + lane_off + C::DS_COL + buf * (T / 2) + col / 2, pk);
+          }
+        }
         // per-token values as 16-byte broadcasts: one shared-memory wavefront per 4 tokens
         const float4* cl4 = reinterpret_cast<const float4*>(cl);
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
+        for (int c = 0; c < 2 && !TW; ++c) {
           const int col = 64 * sw + 32 * c;
           uint32_t pk[16];
 #pragma unroll
@@ -1430,7 +1517,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(ds_full);
-          mbar_arrive(col_empty0 + 8 * buf);
+          if (!TW) mbar_arrive(col_empty0 + 8 * buf);
         }
         // dQ partial of this worker and head (or user segment) at the end of its piece
         const bool more = li + 1 < ntiles;
@@ -1461,6 +1548,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int D, int PS>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                     const __grid_constant__ CUtensorMap tmQ, Args a, const float* __restrict__ dsk,
+                     const float* __restrict__ lse, const float* __restrict__ Dco) {
+  bwd_dq_body<D, PS, false>(tmK, tmV, tmQ, a, dsk, lse, Dco);
+}
+
+template <int D, int PS>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_tw_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                        const __grid_constant__ CUtensorMap tmQ, Args a, const float* __restrict__ dsk,
+                        const float* __restrict__ lse_tok, const float* __restrict__ Dtw) {
+  bwd_dq_body<D, PS, true>(tmK, tmV, tmQ, a, dsk, lse_tok, Dtw);
+}
+
+template <int D, int PS, bool TW = false>
 static cudaError_t launch_dq_t(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
                                cudaStream_t st) {
   using C = QCfg<D, PS>;
@@ -1468,7 +1571,7 @@ static cudaError_t launch_dq_t(const Args& a, int W, const float* dsk, const flo
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
       !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, PS))
     return cudaErrorInvalidValue;
-  auto fn = &tc_bwd_dq_kernel<D, PS>;
+  auto fn = TW ? &tc_tw_bwd_dq_kernel<D, PS> : &tc_bwd_dq_kernel<D, PS>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid(W, a.P / PS);
@@ -1484,5 +1587,28 @@ cudaError_t launch_tc_bwd_dq(const Args& a, int W, const float* dsk, const float
                              cudaStream_t st) {
   if (a.N == 0) return cudaSuccess;
   return tcb::launch_dq_t<128, 128>(a, W, dsk, lse, Dco, st);
+}
+
+// Token-wise normalisation (Sec. 5.1): the same two kernels with per-prototype
+// lse_tok and D_j = G_j . O_j ([B][H][P]); d = 128 and P in {256, ..., 2048}.
+bool tc_tw_bwd_supported(int P, int d, sa_dtype dt) {
+  return dt == SA_BF16 && d == 128 && (P == 256 || P == 512 || P == 1024 || P == 2048) && tcc::device_is_sm103() &&
+         tc_path_enabled();
+}
+
+cudaError_t launch_tc_tw_bwd_tok(const Args& a, int W, const __nv_bfloat16* gbf, const float* lse_tok,
+                                 const float* Dtw, void* dK, void* dV, cudaStream_t st) {
+  if (a.N == 0) return cudaSuccess;
+  float* Dp = const_cast<float*>(Dtw);  // read only in token-wise mode
+  if (a.P == 2048) return tcb::launch_tok_t<128, 2048, true>(a, W, gbf, lse_tok, Dp, dK, dV, st);
+  if (a.P == 1024) return tcb::launch_tok_t<128, 1024, true>(a, W, gbf, lse_tok, Dp, dK, dV, st);
+  if (a.P == 512) return tcb::launch_tok_t<128, 512, true>(a, W, gbf, lse_tok, Dp, dK, dV, st);
+  return tcb::launch_tok_t<128, 256, true>(a, W, gbf, lse_tok, Dp, dK, dV, st);
+}
+
+cudaError_t launch_tc_tw_bwd_dq(const Args& a, int W, const float* dsk, const float* lse_tok, const float* Dtw,
+                                cudaStream_t st) {
+  if (a.N == 0) return cudaSuccess;
+  return tcb::launch_dq_t<128, 128, true>(a, W, dsk, lse_tok, Dtw, st);
 }
 }  // namespace sa

@@ -182,15 +182,21 @@ __global__ void __launch_bounds__(256) tw_finalize_kernel(const void* ws, const 
 }
 
 // D[r] = sum_c G[r, c] O[r, c] for every row r of [B*H*P, d]; one warp per row.
+// With round_g, G is taken rounded to bf16: the tensor-core backward forms
+// dA = G V^T from that rounded copy, and dS = A o (dA - D) cancels exactly
+// only if D is built from the same G (a one-token user has dS = 0).
 __global__ void __launch_bounds__(256) tw_dcoef_kernel(const void* ws, const float* __restrict__ O,
                                                        const float* __restrict__ G, int64_t rows, int d,
-                                                       float* __restrict__ D) {
+                                                       int round_g, float* __restrict__ D) {
   if (ws_failed(ws)) return;
   const int64_t r = int64_t(blockIdx.x) * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
   float s = 0.f;
-  for (int c = lane; c < d; c += 32) s = fmaf(G[r * d + c], O[r * d + c], s);
+  for (int c = lane; c < d; c += 32) {
+    const float g = round_g ? __bfloat162float(__float2bfloat16_rn(G[r * d + c])) : G[r * d + c];
+    s = fmaf(g, O[r * d + c], s);
+  }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   if (lane == 0) D[r] = s;
@@ -409,9 +415,10 @@ cudaError_t launch_tw_finalize(const Args& a, int W, const float2* stat_part, fl
   return cudaGetLastError();
 }
 
-cudaError_t launch_tw_dcoef(const Args& a, const float* O, const float* G, float* D, cudaStream_t st) {
+cudaError_t launch_tw_dcoef(const Args& a, const float* O, const float* G, bool round_g, float* D,
+                            cudaStream_t st) {
   const int64_t rows = int64_t(a.B) * a.H * a.P;
-  tw_dcoef_kernel<<<unsigned((rows + 7) / 8), 256, 0, st>>>(a.ws, O, G, rows, a.d, D);
+  tw_dcoef_kernel<<<unsigned((rows + 7) / 8), 256, 0, st>>>(a.ws, O, G, rows, a.d, round_g ? 1 : 0, D);
   return cudaGetLastError();
 }
 

@@ -161,3 +161,23 @@ def test_tokenwise_growing_scores_rescale(cuda_lib, d):
     got_lse = wl.torch_as_f64(lse)
     fin = np.isfinite(ref_lse)
     assert np.max(np.abs(got_lse[fin] - ref_lse[fin])) <= 5e-5 * max(1.0, np.max(np.abs(ref_lse[fin])))
+
+
+@pytest.mark.parametrize("P", [256, 512, 1024])
+def test_tokenwise_backward_tensor_core_matches_cuda_core(cuda_lib, P):
+    """The tcgen05 backward (token side + prototype slices) against the CUDA-core
+    backward, both fed the same forward outputs."""
+    spec = wl.custom(RAGGED, H=2, P=P, d=128, dtype=wl.BF16, seed=P + 15)
+    host = wl.make_host(spec)
+    t = wl.host_to_torch(spec, host, torch.device("cuda"))
+    args = (t["K"], t["V"], t["cu_seqlens"], t["Q"])
+    O, lse = binding.sa_sketch_fwd_tokenwise(*args, spec.scale, want_lse=True)
+    tc = binding.sa_sketch_bwd_tokenwise(*args, t["dsketch"], spec.scale, sketch=O, lse=lse)
+    binding.sa_select_path(1)
+    try:
+        simt = binding.sa_sketch_bwd_tokenwise(*args, t["dsketch"], spec.scale, sketch=O, lse=lse)
+    finally:
+        binding.sa_select_path(0)
+    torch.cuda.synchronize()
+    for name, x, y in zip(("dK", "dV", "dQ"), tc, simt):
+        assert harness.rel_err(wl.torch_as_f64(x), wl.torch_as_f64(y)) <= 2e-2, name
