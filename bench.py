@@ -285,6 +285,7 @@ def run_ours(args, spec, lens):
     step_w = rf.step_work(tokens, B, H, P, d, eb)
     t_roof = rf.roofline_time(step_w, peak_t, pk["hbm_gbs"])
 
+    tw = tokenwise_leg(args, spec, data, dev, pk) if rank == 0 else None
     e2e = e2e_run(args, spec, dev) if rank == 0 else None
     cpu = oracle_sample(spec, budget_s=15.0) if (rank == 0 and world == 1) else None
 
@@ -299,10 +300,63 @@ def run_ours(args, spec, lens):
                                   "frac": t_roof["time"] * 1e3 / ms_per_step},
                 "roofline": r_bwd, "roofline_fwd": r_fwd,
                 "cpu_baseline": cpu, "e2e": e2e, "clocks": clk.summary(), "gpu_launches": int(launches),
-                "kernels": {"fwd": fwd_name, "bwd": bwd_name}, "kernel_ms": per_kernel}
+                "kernels": {"fwd": fwd_name, "bwd": bwd_name}, "kernel_ms": per_kernel, "tokenwise": tw}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def tokenwise_leg(args, spec, data, dev, pk):
+    """The token-wise normalisation of Sec. 5.1 (weights normalised over each
+    user's tokens) on the same inputs: K fwd+bwd steps through the C ABI, timed
+    like the main step, with its main kernels' rates against the bf16 peak.
+    Reported beside the headline, not part of it."""
+    import torch
+
+    from paper_2609_08443_gb300 import binding
+
+    K, V, Q, cu, dS = data["K"], data["V"], data["Q"], data["cu_seqlens"], data["dsketch"]
+    B = cu.numel() - 1
+    N, H, d = K.shape
+    P = Q.shape[1]
+    tokens = N
+    lib = binding.load()
+    ws = torch.empty(lib.sa_workspace_size_tokenwise(B, N, H, P, d, binding.SA_BF16, 1), dtype=torch.uint8,
+                     device=dev)
+
+    def step():
+        O, lse = binding.sa_sketch_fwd_tokenwise(K, V, cu, Q, spec.scale, want_lse=True, ws=ws)
+        return binding.sa_sketch_bwd_tokenwise(K, V, cu, Q, dS, spec.scale, sketch=O, lse=lse, ws=ws)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    stream = torch.cuda.current_stream(dev)
+    torch.cuda.synchronize(dev)
+    binding.sa_timing_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / args.steps
+    kms = {}
+    for cls, label in ((binding.SA_KERNEL_FWD_MAIN, "fwd_main"), (binding.SA_KERNEL_BWD_MAIN, "bwd_main"),
+                       (binding.SA_KERNEL_BWD_DQ, "bwd_dq")):
+        t, n = binding.sa_timing_read(cls)
+        kms[label] = {"ms_per_call": t / args.steps, "launches": n}
+    binding.sa_timing_enable(False)
+    if binding.sa_get_device_error(ws) != 0:
+        raise RuntimeError("device-side error in the token-wise leg")
+    peak_t = pk["bf16_tflops_sustained"]
+    fw = rf.fwd_work(tokens, B, H, P, d, 2, lse=True)
+    bw = rf.bwd_work(tokens, B, H, P, d, 2, lse_in=True)
+    f_ms = kms["fwd_main"]["ms_per_call"]
+    b_ms = kms["bwd_main"]["ms_per_call"] + kms["bwd_dq"]["ms_per_call"]
+    return {"value": tokens / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms, "kernel_ms": kms,
+            "fwd_tflops": fw.flops / (f_ms / 1e3) / 1e12, "fwd_frac": fw.flops / (f_ms / 1e3) / 1e12 / peak_t,
+            "bwd_tflops": bw.flops / (b_ms / 1e3) / 1e12, "bwd_frac": bw.flops / (b_ms / 1e3) / 1e12 / peak_t,
+            "peak": peak_t, "peak_source": f"{pk['source']} (bf16 sustained)"}
 
 
 def traffic_for(kernel_name):

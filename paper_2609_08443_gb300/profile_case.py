@@ -23,6 +23,7 @@ def main():
     ap.add_argument("--users", type=int, default=4)
     ap.add_argument("--steps", type=int, default=2)
     ap.add_argument("--fwd-only", action="store_true")
+    ap.add_argument("--tokenwise", action="store_true", help="token-wise normalisation (Sec. 5.1) instead")
     args = ap.parse_args()
     spec = wl.config(args.config)
     sub = wl.sub_spec(spec, list(range(min(args.users, spec.B if spec.kind != "extremes" else 4100))))
@@ -30,6 +31,11 @@ def main():
     data = wl.make_device(sub, dev)
     K, V, Q, cu, dS = data["K"], data["V"], data["Q"], data["cu_seqlens"], data["dsketch"]
     for _ in range(args.steps):
+        if args.tokenwise:
+            s, lse = binding.sa_sketch_fwd_tokenwise(K, V, cu, Q, sub.scale, want_lse=True)
+            if not args.fwd_only and spec.bwd:
+                binding.sa_sketch_bwd_tokenwise(K, V, cu, Q, dS, sub.scale, sketch=s, lse=lse)
+            continue
         s, lse = binding.sa_sketch_fwd(K, V, cu, Q, sub.scale, want_lse=True)
         if not args.fwd_only and spec.bwd:
             binding.sa_sketch_bwd(K, V, cu, Q, dS, sub.scale, lse=lse)

@@ -1,7 +1,8 @@
 """DRAM traffic of the tensor-core kernels, from an `ncu` capture of
 `profile_case`, scaled to one call at the full workload size.
 
-    python -m paper_2609_08443_gb300.profile_traffic prof.ncu-rep --config 4 --users 4 > profiles/traffic.json
+    python -m paper_2609_08443_gb300.profile_traffic prof.ncu-rep [more.ncu-rep ...] --config 4 --users 4 \
+        > profiles/traffic.json
 
 The capture runs a sub-batch of `--users` users with the workload's per-user
 shapes; K/V streaming dominates the traffic and grows with the number of
@@ -48,24 +49,27 @@ def kernel_bytes(report: str) -> dict:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("report")
+    ap.add_argument("report", nargs="+", help="ncu reports of profile_case on the same sub-batch")
     ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--users", type=int, default=4)
     args = ap.parse_args()
     spec = wl.config(args.config)
     lens = wl.lengths(spec)
     scale = float(sum(lens)) / float(sum(lens[: args.users]))
-    agg = kernel_bytes(args.report)
+    agg = {}
+    for rep in args.report:
+        agg.update(kernel_bytes(rep))
     h = build.source_hash()
     res = {}
     for name, e in sorted(agg.items()):
         res[name] = {"bytes_per_launch": e["bytes"] / e["launches"] * scale, "captured_launches": e["launches"],
                      "scale": scale, "source_hash": h}
     # the backward's two main kernels count as one call, as the bench times them
-    tok = next((k for k in res if k.startswith("tc_bwd_tok_kernel")), None)
-    dq = next((k for k in res if k.startswith("tc_bwd_dq_kernel")), None)
-    if tok and dq:
-        res[tok]["bytes_per_call"] = res[tok]["bytes_per_launch"] + res[dq]["bytes_per_launch"]
+    for tok_pre, dq_pre in (("tc_bwd_tok_kernel", "tc_bwd_dq_kernel"), ("tc_tw_bwd_tok_kernel", "tc_tw_bwd_dq_kernel")):
+        tok = next((k for k in res if k.startswith(tok_pre)), None)
+        dq = next((k for k in res if k.startswith(dq_pre)), None)
+        if tok and dq:
+            res[tok]["bytes_per_call"] = res[tok]["bytes_per_launch"] + res[dq]["bytes_per_launch"]
     for name in res:
         res[name].setdefault("bytes_per_call", res[name]["bytes_per_launch"])
     json.dump(res, sys.stdout, indent=1, sort_keys=True)
