@@ -628,6 +628,14 @@ struct TokCfg {
   static_assert(NC == T && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
 };
 
+// Where dA lands: with prototype-wise weights S and dA share SD_COL (TMEM is
+// full); token-wise needs no qbar, so dA takes QB_COL and the two do not wait
+// for each other.
+template <int D, int P, bool TW>
+__host__ __device__ constexpr int tok_da_col() {
+  return TW ? TokCfg<D, P>::QB_COL : TokCfg<D, P>::SD_COL;
+}
+
 // Pair 0 holds the tile's K and V; the next tile's K loads into it once the
 // tile's last S has read K, its V once the last dA has read V, and both tiles
 // are pulled into L2 a tile ahead.  Chunks alternate between pairs 1 and 2
@@ -793,17 +801,20 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
         const int li = int(g / C::NCH), c = int(g % C::NCH);
         const int kvp = tok_kv_pair(li), qgp = tok_qg_pair(li, c);
         const uint32_t aG = slot_addr(2 * qgp), aQ = slot_addr(2 * qgp + 1);
-        // ---- dA_g = V G_g^T
+        // ---- dA_g = V G_g^T (into S's columns once S_g is read, or, token-wise,
+        // into its own columns once dA_{g-1} is read)
         if (c == 0) wfull(2 * kvp + 1, 0x903);
         wfull(2 * qgp, 0x904);
-        wt(sd_free_s, g & 1, 0x905);
+        if (!TW) wt(sd_free_s, g & 1, 0x905);
+        else if (g > 0) wt(sd_free_da, (g - 1) & 1, 0x905);
         if (!ok) break;
         tc_fence_after();
         {
           const uint64_t dV = kmaj(slot_addr(2 * kvp + 1)), dG = kmaj(aG);
 #pragma unroll
           for (int k = 0; k < D / 16; ++k)
-            umma_ss(tmem + C::SD_COL, sdesc_add(dV, kstep(k)), sdesc_add(dG, kstep(k)), idS, k > 0 ? 1u : 0u);
+            umma_ss(tmem + tok_da_col<D, P, TW>(), sdesc_add(dV, kstep(k)), sdesc_add(dG, kstep(k)), idS,
+                    k > 0 ? 1u : 0u);
         }
         umma_commit(da_full);
         if (c == C::NCH - 1) umma_commit(empty_bar(2 * kvp + 1));  // last dA: V free
@@ -827,7 +838,7 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
           const int lin = int(gn / C::NCH), cn = int(gn % C::NCH);
           if (cn == 0) wfull(2 * tok_kv_pair(lin), 0x908);
           wfull(2 * tok_qg_pair(lin, cn) + 1, 0x909);
-          wt(sd_free_da, g & 1, 0x90A);
+          wt(TW ? sd_free_s : sd_free_da, g & 1, 0x90A);  // S's columns read
           if (!ok) break;
           tc_fence_after();
           issue_S(gn);
@@ -955,7 +966,7 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
           uint32_t epk[C::HALF / 2];
 #pragma unroll
           for (int cc = 0; cc < C::HALF / 32; ++cc) {
-            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * cc, v);
+            tmem_ld32(tmem + lane_off + tok_da_col<D, P, TW>() + sw * C::HALF + 32 * cc, v);
             tmem_ld_wait();
             if (TW) {
               const float4* d4 = reinterpret_cast<const float4*>(Dco + seg_row + j0 + 32 * cc);
