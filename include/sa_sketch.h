@@ -170,6 +170,35 @@ sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* c
                                   const float* dsketch, void* dK, void* dV, float* dQ,
                                   void* workspace, size_t ws_bytes, void* stream);
 
+/* The training step (forward and backward, Sec. 3.1) on a batch held in HOST
+ * memory (the paper has no counterpart; a runtime convenience).  K, V, Q and
+ * dsketch are host arrays, sketch, dK, dV and dQ host arrays the call fills;
+ * shapes, dtypes and the results are those of sa_sketch_fwd followed by
+ * sa_sketch_bwd (lse is kept internal).  cu_seqlens_host is a host array.
+ *   - Users are grouped into chunks of at most chunk_tokens tokens (<= 0: 262144;
+ *     a longer user is a chunk of its own; at most 1024 users per chunk).  Three
+ *     internal streams overlap the host-to-device copy of a chunk, the step on
+ *     the previous chunk and the device-to-host copy of the one before; dQ is
+ *     summed over the chunks in chunk order (bitwise reproducible for a given
+ *     chunk_tokens, but not bitwise equal to one sa_sketch_bwd call on the
+ *     whole batch: the summation groups differ).
+ *   - Asynchronous with respect to the host: the call enqueues everything and
+ *     makes `stream` wait for it, so synchronising `stream` means the host
+ *     outputs are written.  Page-locked host arrays give overlapped copies;
+ *     pageable ones are correct but serialise the copies.  Host arrays must stay
+ *     valid and unchanged until then.
+ *   - `workspace` is device memory of sa_step_host_workspace_size() bytes
+ *     (256-byte aligned); sa_get_device_error(workspace, stream) reports the
+ *     first device-detected error of any chunk.
+ *   - Not thread-safe: the pipeline's streams are shared per device; serialise
+ *     calls on one device. */
+size_t sa_step_host_workspace_size(const int32_t* cu_seqlens_host, int B, int H, int P, int d, sa_dtype dt,
+                                   int64_t chunk_tokens);
+sa_status sa_sketch_step_host(const void* K, const void* V, const int32_t* cu_seqlens_host, int B,
+                              int64_t N, const void* Q, int H, int P, int d, float scale, sa_dtype dt,
+                              const float* dsketch, float* sketch, void* dK, void* dV, float* dQ,
+                              int64_t chunk_tokens, void* workspace, size_t ws_bytes, void* stream);
+
 /* Allocation-free forward (the paper has no counterpart; this is a library
  * convenience).  For callers that cannot provide a workspace: for example a
  * plugin or custom-operator hook that receives only its input and output
@@ -248,6 +277,11 @@ const char* sa_main_kernel_name(int P, int d, sa_dtype dt, int bwd);
  * from host cu_seqlens; returns SA_ERR_BAD_SEQLENS for invalid offsets. */
 sa_status sa_plan_host(const int32_t* cu_seqlens_host, int B, int H, int tile, int n_workers,
                        int64_t* begin);
+
+/* The chunks sa_sketch_step_host forms: users [begin[c], begin[c+1]) are chunk
+ * c, for c < *n_chunks; `begin` must hold B + 1 entries. */
+sa_status sa_plan_chunks_host(const int32_t* cu_seqlens_host, int B, int64_t chunk_tokens, int* begin,
+                              int* n_chunks);
 
 #ifdef __cplusplus
 }

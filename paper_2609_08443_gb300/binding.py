@@ -83,6 +83,13 @@ def load() -> ctypes.CDLL:
     lib.sa_sketch_bwd_tokenwise.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp, vp, vp,
                                             vp, vp, sz, vp]
     lib.sa_sketch_bwd_tokenwise.restype = i32
+    lib.sa_step_host_workspace_size.argtypes = [vp, i32, i32, i32, i32, i32, i64]
+    lib.sa_step_host_workspace_size.restype = sz
+    lib.sa_sketch_step_host.argtypes = [vp, vp, vp, i32, i64, vp, i32, i32, i32, f32, i32, vp, vp, vp, vp, vp, i64,
+                                        vp, sz, vp]
+    lib.sa_sketch_step_host.restype = i32
+    lib.sa_plan_chunks_host.argtypes = [vp, i32, i64, vp, vp]
+    lib.sa_plan_chunks_host.restype = i32
     lib.sa_plan_host.argtypes = [vp, i32, i32, i32, i32, vp]
     lib.sa_plan_host.restype = i32
     _lib = lib
@@ -395,6 +402,58 @@ def sa_sketch_bwd_tokenwise(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.
                                      _ptr(w), w.numel(), _stream(K.device))
     _check(st, "sa_sketch_bwd_tokenwise")
     return dK, dV, dQ
+
+
+def sa_sketch_step_host(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Tensor, Q: torch.Tensor,
+                        dsketch: torch.Tensor, scale: Optional[float] = None, chunk_tokens: int = 0,
+                        outs=None, device=None, ws: Optional[torch.Tensor] = None):
+    """Forward + backward of a batch held in host memory (C: sa_sketch_step_host):
+    K, V [N,H,d], cu_seqlens [B+1] int32, Q [H,P,d], dsketch [B,H,P,d] fp32, all
+    CPU tensors (page-locked for overlapped copies).  Returns CPU tensors
+    (sketch, dK, dV, dQ), written once the current stream of ``device`` is
+    synchronised (this function synchronises it before returning)."""
+    lib = load()
+    for name, t in (("K", K), ("V", V), ("Q", Q), ("cu_seqlens", cu_seqlens), ("dsketch", dsketch)):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CPU tensor")
+    N, H, d = K.shape
+    P = Q.shape[1]
+    B = cu_seqlens.numel() - 1
+    if cu_seqlens.dtype != torch.int32 or V.shape != K.shape or tuple(Q.shape) != (H, P, d) or \
+            tuple(dsketch.shape) != (B, H, P, d) or dsketch.dtype != torch.float32:
+        raise ValueError("shapes: K,V [N,H,d], Q [H,P,d], cu_seqlens int32 [B+1], dsketch fp32 [B,H,P,d]")
+    dt = _dt(K)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    if outs is None:
+        pin = K.is_pinned()
+        outs = (torch.empty((B, H, P, d), dtype=torch.float32, pin_memory=pin),
+                torch.empty_like(K, pin_memory=pin), torch.empty_like(V, pin_memory=pin),
+                torch.empty((H, P, d), dtype=torch.float32, pin_memory=pin))
+    sketch, dK, dV, dQ = outs
+    need = lib.sa_step_host_workspace_size(_ptr(cu_seqlens), B, H, P, d, dt, int(chunk_tokens))
+    if need == 0:
+        raise SketchError(2, "sa_step_host_workspace_size")
+    w = ws if ws is not None else workspace(need, dev)
+    st = lib.sa_sketch_step_host(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, dt,
+                                 _ptr(dsketch), _ptr(sketch), _ptr(dK), _ptr(dV), _ptr(dQ), int(chunk_tokens),
+                                 _ptr(w), w.numel(), _stream(dev))
+    _check(st, "sa_sketch_step_host")
+    torch.cuda.current_stream(dev).synchronize()
+    return sketch, dK, dV, dQ
+
+
+def sa_plan_chunks_host(cu_seqlens_host, chunk_tokens: int = 0):
+    """Chunk boundaries (user indices) sa_sketch_step_host uses (pure C; no GPU)."""
+    import numpy as np
+
+    cu = np.ascontiguousarray(cu_seqlens_host, dtype=np.int32)
+    begin = np.zeros(cu.size, dtype=np.int32)
+    n = ctypes.c_int()
+    st = load().sa_plan_chunks_host(cu.ctypes.data, cu.size - 1, int(chunk_tokens), begin.ctypes.data,
+                                    ctypes.byref(n))
+    _check(st, "sa_plan_chunks_host")
+    return begin[: n.value + 1]
 
 
 def sa_noalloc_scratch_bytes() -> int:

@@ -120,3 +120,35 @@ def test_tokenwise_host_checks(lib):
     b = binding.load().sa_workspace_size_tokenwise(4, 1000, 2, 256, 64, 1, 1)
     assert a > 0 and b > a and a % 256 == 0 and b % 256 == 0
     assert binding.load().sa_workspace_size_tokenwise(1, 10, 1, 4096, 64, 1, 0) == 0
+
+
+def test_chunk_plan_host(lib):
+    """The user chunks of the host-buffer pipeline: consecutive users within the
+    token budget, a longer user alone, every user exactly once."""
+    lens = [5, 0, 7, 3, 20, 1, 1, 0, 6]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    b = binding.sa_plan_chunks_host(cu, chunk_tokens=10)
+    assert b[0] == 0 and b[-1] == len(lens) and np.all(np.diff(b) > 0)
+    for c in range(len(b) - 1):
+        tok = int(cu[b[c + 1]] - cu[b[c]])
+        assert tok <= 10 or b[c + 1] - b[c] == 1, (c, tok)
+        if c + 1 < len(b) - 1:  # a chunk closes only when the next user would overflow it
+            assert tok + lens[b[c + 1]] > 10
+    assert list(b) == [0, 2, 4, 5, 9]
+    many = np.arange(3001, dtype=np.int32)  # 3000 one-token users: at most 1024 per chunk
+    assert list(binding.sa_plan_chunks_host(many, chunk_tokens=1 << 20)) == [0, 1024, 2048, 3000]
+    with pytest.raises(binding.SketchError):
+        binding.sa_plan_chunks_host(np.array([0, 5, 3], dtype=np.int32))
+
+
+def test_step_host_checks(lib):
+    vp = ctypes.c_void_p
+    cu = np.array([0, 4, 10], dtype=np.int32)
+    # NULL host output and a workspace that is too small: refused before any copy
+    st = lib.sa_sketch_step_host(vp(256), vp(512), cu.ctypes.data, 2, 10, vp(1024), 1, 64, 64, 0.125, 1, vp(2048),
+                                 None, vp(4096), vp(8192), vp(9216), 0, vp(1 << 20), 1 << 30, None)
+    assert st == 1
+    st = lib.sa_sketch_step_host(vp(256), vp(512), cu.ctypes.data, 2, 10, vp(1024), 1, 64, 64, 0.125, 1, vp(2048),
+                                 vp(3072), vp(4096), vp(8192), vp(9216), 0, vp(1 << 20), 16, None)
+    assert st == 3
+    assert lib.sa_step_host_workspace_size(cu.ctypes.data, 2, 1, 64, 64, 1, 0) > 0
