@@ -169,6 +169,21 @@ def run_reference(args, spec, lens):
 
 # ------------------------------------------------------------------- GPU arm
 
+def job_rate(ms_local, tokens_per_rank, steps, world, device):
+    """Whole-job timing of N ranks that each processed `tokens_per_rank` tokens
+    per step for `steps` steps: the slowest rank's time (all-reduce MAX; each
+    rank is an independent replica, so this is the only collective) and the
+    job's tokens/s over it.  Returns (ms, tokens/s), the same on every rank."""
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(ms_local)], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms = float(t.item())
+    return ms, tokens_per_rank * world * steps / (ms / 1e3)
+
+
 def run_ours(args, spec, lens):
     import torch
     import torch.distributed as dist
@@ -246,12 +261,8 @@ def run_ours(args, spec, lens):
     binding.sa_timing_enable(False)
     if binding.sa_get_device_error(ws) != 0:
         raise RuntimeError("device-side error in the timed region")
-    t_max = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
-    ms = float(t_max.item())
+    ms, value = job_rate(ms, tokens, args.steps, world, dev)
     ms_per_step = ms / args.steps
-    value = tokens * world * args.steps / (ms / 1e3)
 
     # roofline of the dominant kernel (the backward main kernel) and of the forward
     eb = 2
