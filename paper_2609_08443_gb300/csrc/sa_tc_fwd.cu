@@ -43,6 +43,9 @@ using namespace tcc;
 
 enum Mode { kFused = 0, kSliced = 1, kPair = 2 };
 
+constexpr uint32_t kRegsCtl = 104, kRegsSoft = 200;
+static_assert(128 * kRegsCtl + 256 * kRegsSoft == 384 * 168, "register split = launch allocation");
+
 template <int D, int PS, int MODE>
 struct Cfg {
   static constexpr int KV_TILE = T * D * 2;
@@ -146,7 +149,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (ntiles > 0) {
+  // Registers: the control warpgroup (warps 0-3) gives up registers so that the
+  // two softmax warpgroups can hold a tile row of 128 scores without spilling:
+  // 128 x kRegsCtl + 256 x kRegsSoft = 384 x 168, the launch allocation.
+  if (ntiles > 0 && warp < kSoftWarp0) {
+    setmaxnreg_dec<kRegsCtl>();
     if (warp == 0 && lane == 0) {
       // ------------------------------------------------------ TMA producer
       tma_prefetch_desc(&tmK);
@@ -298,7 +305,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       // make sure no UMMA is still running when TMEM is released
       umma_commit(drain);
       mbar_wait_bounded(drain, 0, 200000000ull);
-    } else if (warp >= kSoftWarp0) {
+    }
+  } else if (ntiles > 0) {
+    setmaxnreg_inc<kRegsSoft>();
+    {
       // ------------------------------------------- softmax + epilogue warps
       const int sw = (warp - kSoftWarp0) >> 2;  // warpgroup: prototype half
       const int q = warp & 3;                   // TMEM lane quadrant

@@ -114,7 +114,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (ntiles > 0) {
+  // Registers: the control warpgroup (warps 0-3) hands registers to the two
+  // softmax warpgroups, which hold a row of 128 scores (128 x 88 + 256 x 208 =
+  // 384 x 168, the launch allocation).
+  if (ntiles > 0 && warp < kSoftWarp0) {
+    setmaxnreg_dec<88>();
     if (warp == 0 && lane == 0) {
       // ------------------------------------------------------ TMA producer
       // K of tile li and V of tile li - 1 alternate in one ring of slots
@@ -260,7 +264,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       umma_commit(drain);  // no UMMA may still run when TMEM is released
       mbar_wait_bounded(drain, 0, 200000000ull);
-    } else if (warp >= kSoftWarp0 && warp < kSoftWarp0 + C::SOFT_WARPS) {
+    }
+  } else if (ntiles > 0) {
+    setmaxnreg_inc<208>();
+    if (warp < kSoftWarp0 + C::SOFT_WARPS) {
       // ------------------------------------------- softmax + epilogue warps
       const int g = (warp - kSoftWarp0) >> 2;  // M-tile
       const int q = warp & 3;                  // TMEM lane quadrant
