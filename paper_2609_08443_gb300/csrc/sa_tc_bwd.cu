@@ -720,14 +720,19 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
       TileWalker it(a, tb, te, T), nx(a, tb, te, T);
       nx.next();
       static_assert(C::NCH % 2 == 0, "chunks alternate between two pairs");
-      int uses[C::NSLOT] = {0, 0, 0, 0, 0, 0};
+      // per slot, as bits (registers, not an indexed array): loaded before, and
+      // the parity of the wait for its next release
+      uint32_t used = 0u, par = 0u;
       bool ok = true;
       // box origin (64*dh, c1, c2): K / V maps are (d, head, token); Q / G maps
       // are (d, prototype, head) and (d, prototype, user*H + head)
       auto load = [&](int s, const CUtensorMap* map, int c1, int c2) {
-        if (uses[s] > 0) ok = ok && mbar_wait(empty_bar(s), (uses[s] - 1) & 1, abort_flag, a.ws, 0x801);
+        if ((used >> s) & 1u) {
+          ok = ok && mbar_wait(empty_bar(s), (par >> s) & 1u, abort_flag, a.ws, 0x801);
+          par ^= 1u << s;
+        }
         if (!ok) return;
-        ++uses[s];
+        used |= 1u << s;
         mbar_arrive_expect_tx(full_bar(s), C::SLOT);
 #pragma unroll
         for (int dh = 0; dh < D / 64; ++dh) tma_load_3d(slot_addr(s) + dh * T * 128, map, full_bar(s), 64 * dh, c1, c2);
@@ -758,7 +763,7 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
       }
       if (!ok) {
         for (int s = 0; s < C::NSLOT; ++s)
-          if (uses[s] > 0) mbar_wait_bounded(full_bar(s), (uses[s] - 1) & 1, 200000000ull);
+          if ((used >> s) & 1u) mbar_wait_bounded(full_bar(s), (par >> s) & 1u, 200000000ull);
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- UMMA issuer
@@ -769,13 +774,13 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
       constexpr uint32_t idGQ = idesc_bf16(128, TW ? D : 2 * D, 0, 1);  // [tok x (d | d)] (TW: d), K = chunk
       constexpr uint32_t idU = idesc_bf16(128, D, 0, 1);        // [tok x d], K = chunk prototypes
       bool ok = true;
-      int uses[C::NSLOT] = {0, 0, 0, 0, 0, 0};
-      auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
-        return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
+      uint32_t fpar = 0u;  // per slot, as bits: parity of the next "full" phase
+      auto wt = [&](uint32_t bar, uint32_t parity, uint32_t site) {
+        return ok = ok && mbar_wait(bar, parity, abort_flag, a.ws, site);
       };
       auto wfull = [&](int s, uint32_t site) {
-        wt(full_bar(s), uses[s] & 1, site);
-        ++uses[s];
+        wt(full_bar(s), (fpar >> s) & 1u, site);
+        fpar ^= 1u << s;
       };
       // K-major [128 rows x D] operand: K step k at +(k / 4) * 128 rows + (k % 4) * 32 B
       auto kmaj = [](uint32_t addr) { return sdesc(addr, 16, 1024); };
