@@ -710,7 +710,10 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (ntiles > 0) {
+  // Registers: the control warpgroup (warps 0-3) hands registers to the two
+  // softmax warpgroups (128 x 152 + 256 x 176 = 384 x 168, the launch allocation).
+  if (ntiles > 0 && warp < kSoftWarp0) {
+    setmaxnreg_dec<152>();
     if (warp == 0 && lane == 0) {
       // ---------------------------------------------------------- TMA producer
       tma_prefetch_desc(&tmK);
@@ -865,7 +868,10 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
       }
       umma_commit(drain);
       mbar_wait_bounded(drain, 0, 200000000ull);
-    } else if (warp >= kSoftWarp0) {
+    }
+  } else if (ntiles > 0) {
+    setmaxnreg_inc<176>();
+    {
       // ------------------------------------------------ softmax + epilogue
       const int sw = (warp - kSoftWarp0) >> 2, q = warp & 3, row = 32 * q + lane;
       const uint32_t lane_off = uint32_t(32 * q) << 16;
@@ -923,39 +929,41 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
         float Dp = 0.f;
         for (int c = 0; c < C::NCH && ok; ++c, ++g) {
           uint32_t apk[C::HALF / 2];
-          float v[32];
+          float v[C::HALF];  // this warpgroup's columns of S, then of dA (both loads before one wait)
           const int j0 = c * C::NC + sw * C::HALF;  // first prototype of this warpgroup's columns
           ok = wwait(s_full, g & 1, 0xA01);
           if (!ok) break;
           tc_fence_after();
 #pragma unroll
+          for (int cc = 0; cc < C::HALF / 32; ++cc) tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * cc, v + 32 * cc);
+          tmem_ld_wait();
+          // S is in registers: its columns may take dA_g (or S_{g+1}) while the weights are formed
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sd_free_s);
+#pragma unroll
           for (int cc = 0; cc < C::HALF / 32; ++cc) {
-            tmem_ld32(tmem + lane_off + C::SD_COL + sw * C::HALF + 32 * cc, v);
-            tmem_ld_wait();
             if (TW) {
               const float4* l4 = reinterpret_cast<const float4*>(lse + seg_row + j0 + 32 * cc);
 #pragma unroll
               for (int j4 = 0; j4 < 8; ++j4) {
                 const float4 l = __ldg(l4 + j4);
-                const float x0 = valid ? ex2(fmaf(v[4 * j4 + 0], c2, -l.x * 1.4426950408889634f)) : 0.f;
-                const float x1 = valid ? ex2(fmaf(v[4 * j4 + 1], c2, -l.y * 1.4426950408889634f)) : 0.f;
-                const float x2 = valid ? ex2(fmaf(v[4 * j4 + 2], c2, -l.z * 1.4426950408889634f)) : 0.f;
-                const float x3 = valid ? ex2(fmaf(v[4 * j4 + 3], c2, -l.w * 1.4426950408889634f)) : 0.f;
+                const float x0 = valid ? ex2(fmaf(v[32 * cc + 4 * j4 + 0], c2, -l.x * 1.4426950408889634f)) : 0.f;
+                const float x1 = valid ? ex2(fmaf(v[32 * cc + 4 * j4 + 1], c2, -l.y * 1.4426950408889634f)) : 0.f;
+                const float x2 = valid ? ex2(fmaf(v[32 * cc + 4 * j4 + 2], c2, -l.z * 1.4426950408889634f)) : 0.f;
+                const float x3 = valid ? ex2(fmaf(v[32 * cc + 4 * j4 + 3], c2, -l.w * 1.4426950408889634f)) : 0.f;
                 apk[16 * cc + 2 * j4] = pack_bf16(x0, x1);
                 apk[16 * cc + 2 * j4 + 1] = pack_bf16(x2, x3);
               }
             } else {
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
-                const float x0 = valid ? ex2(fmaf(v[2 * j], c2, -L2)) : 0.f;
-                const float x1 = valid ? ex2(fmaf(v[2 * j + 1], c2, -L2)) : 0.f;
+                const float x0 = valid ? ex2(fmaf(v[32 * cc + 2 * j], c2, -L2)) : 0.f;
+                const float x1 = valid ? ex2(fmaf(v[32 * cc + 2 * j + 1], c2, -L2)) : 0.f;
                 apk[16 * cc + j] = pack_bf16(x0, x1);
               }
             }
           }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(sd_free_s);
           if (g > 0) {
             ok = wwait(ab_free_e, (g - 1) & 1, 0xA02);  // u of the previous chunk has read E
             if (!ok) break;
@@ -970,33 +978,35 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
           tc_fence_after();
           uint32_t epk[C::HALF / 2];
 #pragma unroll
+          for (int cc = 0; cc < C::HALF / 32; ++cc)
+            tmem_ld32(tmem + lane_off + tok_da_col<D, P, TW>() + sw * C::HALF + 32 * cc, v + 32 * cc);
+          tmem_ld_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sd_free_da);
+#pragma unroll
           for (int cc = 0; cc < C::HALF / 32; ++cc) {
-            tmem_ld32(tmem + lane_off + tok_da_col<D, P, TW>() + sw * C::HALF + 32 * cc, v);
-            tmem_ld_wait();
             if (TW) {
               const float4* d4 = reinterpret_cast<const float4*>(Dco + seg_row + j0 + 32 * cc);
 #pragma unroll
               for (int j4 = 0; j4 < 8; ++j4) {
                 const float4 dd = __ldg(d4 + j4);
                 const uint32_t w0 = apk[16 * cc + 2 * j4], w1 = apk[16 * cc + 2 * j4 + 1];
-                epk[16 * cc + 2 * j4] = pack_bf16(bf16lo(w0) * (v[4 * j4 + 0] - dd.x),
-                                                  bf16hi(w0) * (v[4 * j4 + 1] - dd.y));
-                epk[16 * cc + 2 * j4 + 1] = pack_bf16(bf16lo(w1) * (v[4 * j4 + 2] - dd.z),
-                                                      bf16hi(w1) * (v[4 * j4 + 3] - dd.w));
+                epk[16 * cc + 2 * j4] = pack_bf16(bf16lo(w0) * (v[32 * cc + 4 * j4 + 0] - dd.x),
+                                                  bf16hi(w0) * (v[32 * cc + 4 * j4 + 1] - dd.y));
+                epk[16 * cc + 2 * j4 + 1] = pack_bf16(bf16lo(w1) * (v[32 * cc + 4 * j4 + 2] - dd.z),
+                                                      bf16hi(w1) * (v[32 * cc + 4 * j4 + 3] - dd.w));
               }
             } else {
 #pragma unroll
               for (int j = 0; j < 16; ++j) {
                 const uint32_t w = apk[16 * cc + j];
-                const float e0 = bf16lo(w) * v[2 * j], e1 = bf16hi(w) * v[2 * j + 1];
+                const float e0 = bf16lo(w) * v[32 * cc + 2 * j], e1 = bf16hi(w) * v[32 * cc + 2 * j + 1];
                 Dp += e0 + e1;
                 epk[16 * cc + j] = pack_bf16(e0, e1);
               }
             }
           }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(sd_free_da);
           ok = wwait(ab_free_a, g & 1, 0xA04);  // dV and qbar have read A
           if (!ok) break;
           put_tile(epk);
