@@ -75,7 +75,8 @@ size_t sa_workspace_size(int B, int64_t N, int H, int P, int d, sa_dtype dt, int
 /* Forward: sketch[b,h] = softmax_proto(scale * Q[h] K_b[:,h]^T) V_b[:,h]
  * (Sec. 3.1).  `lse` may be NULL; when given it receives, per token and head,
  * log sum_j exp(S[j,i]) (the softmax statistic FlashSA keeps, Sec. 4.4) so the
- * backward can skip recomputing it.  `scale` is normally 1/sqrt(d). */
+ * backward can skip recomputing it.  `scale` is normally 1/sqrt(d); a negative
+ * scale is valid and runs on the CUDA-core kernels. */
 sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens, int B,
                         int64_t N, const void* Q, int H, int P, int d, float scale,
                         sa_dtype dt, float* sketch, float* lse, void* workspace,

@@ -92,11 +92,14 @@ bool shape_ok(int B, int64_t N, int H, int P, int d, sa_dtype dt) {
   return d % (dt == SA_BF16 ? 8 : 4) == 0;
 }
 
-Plan make_plan(int B, int64_t N, int H, int P, int d, sa_dtype dt, bool bwd) {
+// allow_tc = false keeps every kernel on the CUDA cores: the tensor-core
+// kernels take the softmax maximum on the raw scores, which is the maximum of
+// the scaled scores only for scale >= 0.
+Plan make_plan(int B, int64_t N, int H, int P, int d, sa_dtype dt, bool bwd, bool allow_tc = true) {
   Plan p{};
   const int sms = device_sms() > 0 ? device_sms() : 1;
-  p.fwd_path = sa::tc_fwd_supported(P, d, dt) ? Path::TcFwd : Path::Simt;
-  p.bwd_path = sa::tc_bwd_supported(P, d, dt) ? Path::TcBwd : Path::Simt;
+  p.fwd_path = allow_tc && sa::tc_fwd_supported(P, d, dt) ? Path::TcFwd : Path::Simt;
+  p.bwd_path = allow_tc && sa::tc_bwd_supported(P, d, dt) ? Path::TcBwd : Path::Simt;
   if (p.fwd_path == Path::TcFwd) {
     p.T_fwd = sa::tc_tile_tokens();
     p.W_fwd = sa::tc_fwd_workers(sms, P, d);
@@ -135,7 +138,7 @@ sa_status check_common(const void* K, const void* V, const int32_t* cu, int B, i
                        int H, int P, int d, float scale, sa_dtype dt, const void* ws, size_t ws_bytes,
                        bool bwd, Plan* plan) {
   SA_TRY(check_args(K, V, cu, B, N, Q, H, P, d, scale, dt, ws));
-  *plan = make_plan(B, N, H, P, d, dt, bwd);
+  *plan = make_plan(B, N, H, P, d, dt, bwd, scale >= 0.f);
   if (ws_bytes < plan->lay.total) return SA_ERR_WORKSPACE;
   return SA_OK;
 }
@@ -239,7 +242,10 @@ extern "C" {
 
 size_t sa_workspace_size(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd) {
   if (!shape_ok(B, N, H, P, d, dt)) return 0;
-  return make_plan(B, N, H, P, d, dt, bwd != 0).lay.total;
+  // enough for either plan (a negative scale runs on the CUDA cores)
+  const size_t tc = make_plan(B, N, H, P, d, dt, bwd != 0, true).lay.total;
+  const size_t cc = make_plan(B, N, H, P, d, dt, bwd != 0, false).lay.total;
+  return tc > cc ? tc : cc;
 }
 
 }  // extern "C"

@@ -84,3 +84,34 @@ def test_large_p_100k_user(cuda_lib):
     one 100K-token user, H=8, d=128, P=1024, Q ~ N(0, 0.02), bf16."""
     spec = wl.custom([100000], H=8, P=1024, d=128, dtype=wl.BF16, seed=41, q_std=0.02)
     harness.check_spec(spec, bwd=True)
+
+
+@pytest.mark.parametrize("P,d", [(512, 128), (256, 64)])
+def test_negative_scale(cuda_lib, P, d):
+    """A negative scale (valid; the softmax then favours anti-aligned keys) runs on
+    the CUDA-core kernels: same parity bar."""
+    spec = wl.custom(RAGGED, H=2, P=P, d=d, dtype=wl.BF16, seed=P + d + 5)
+    host = wl.make_host(spec)
+    t = wl.host_to_torch(spec, host, torch.device("cuda"))
+    from paper_2609_08443_gb300 import binding
+    from oracle import sa_backward, sa_forward
+
+    scale = -2.0 / np.sqrt(d)
+    sk, lse = binding.sa_sketch_fwd(t["K"], t["V"], t["cu_seqlens"], t["Q"], scale, want_lse=True)
+    dK, dV, dQ = binding.sa_sketch_bwd(t["K"], t["V"], t["cu_seqlens"], t["Q"], t["dsketch"], scale, lse=lse)
+    dK2, dV2, dQ2 = binding.sa_sketch_bwd(t["K"], t["V"], t["cu_seqlens"], t["Q"], t["dsketch"], scale)
+    torch.cuda.synchronize()
+    K, V, Q = (wl.host_as_f64(spec, host[k]) for k in ("K", "V", "Q"))
+    O, l_ref = sa_forward(K, V, host["cu_seqlens"], Q, scale, with_lse=True)
+    gK, gV, gQ = sa_backward(K, V, host["cu_seqlens"], Q, scale, host["dsketch"].astype(np.float64))
+    tol = harness.TOL[wl.BF16]
+    for name, got, ref in (("sketch", sk, O), ("dK", dK, gK), ("dV", dV, gV), ("dQ", dQ, gQ), ("dK (lse recomputed)", dK2, gK),
+                           ("dQ (lse recomputed)", dQ2, gQ)):
+        harness.assert_close(name, wl.torch_as_f64(got), ref, tol)
+    assert np.max(np.abs(wl.torch_as_f64(lse) - l_ref)) <= 5e-3 * max(1.0, np.max(np.abs(l_ref)))
+
+
+def test_max_heads(cuda_lib):
+    """H = 64, the largest head count, on the tensor-core path."""
+    spec = wl.custom([300, 0, 129, 17, 1000], H=64, P=128, d=64, dtype=wl.BF16, seed=64)
+    harness.check_spec(spec, bwd=True)

@@ -181,3 +181,21 @@ def test_tokenwise_backward_tensor_core_matches_cuda_core(cuda_lib, P):
     torch.cuda.synchronize()
     for name, x, y in zip(("dK", "dV", "dQ"), tc, simt):
         assert harness.rel_err(wl.torch_as_f64(x), wl.torch_as_f64(y)) <= 2e-2, name
+
+
+def test_tokenwise_negative_scale(cuda_lib):
+    """A negative scale runs the token-wise forward on the CUDA cores."""
+    spec = wl.custom(RAGGED, H=2, P=256, d=128, dtype=wl.BF16, seed=17)
+    host = wl.make_host(spec)
+    t = wl.host_to_torch(spec, host, torch.device("cuda"))
+    scale = -1.5 / np.sqrt(128)
+    O, lse = binding.sa_sketch_fwd_tokenwise(t["K"], t["V"], t["cu_seqlens"], t["Q"], scale, want_lse=True)
+    dK, dV, dQ = binding.sa_sketch_bwd_tokenwise(t["K"], t["V"], t["cu_seqlens"], t["Q"], t["dsketch"], scale,
+                                                 sketch=O, lse=lse)
+    torch.cuda.synchronize()
+    K, V, Q = (wl.host_as_f64(spec, host[k]) for k in ("K", "V", "Q"))
+    ref_O = sa_forward_tokenwise(K, V, host["cu_seqlens"], Q, scale)
+    rK, rV, rQ = sa_backward_tokenwise(K, V, host["cu_seqlens"], Q, scale, host["dsketch"].astype(np.float64))
+    tol = harness.TOL[wl.BF16]
+    for name, got, ref in (("sketch", O, ref_O), ("dK", dK, rK), ("dV", dV, rV), ("dQ", dQ, rQ)):
+        harness.assert_close(name, wl.torch_as_f64(got), ref, tol)
