@@ -28,6 +28,7 @@
 // Warp roles: 0 = TMA producer, 1 = UMMA issuer, 2 = TMEM allocator,
 // 4..11 = softmax + epilogue.  Every wait is bounded (sa_ptx.cuh).
 #include <cuda.h>
+#include <cuda_fp16.h>
 
 #include <cstdio>
 
@@ -52,7 +53,11 @@ struct Cfg {
   static constexpr int Q_BYTES = PS * D * 2;
   static constexpr int W_BYTES = T * PS * 2;
   static constexpr int NSLOT = (D == 128) ? 3 : 6;
-  static constexpr int STATS = (MODE == kSliced) ? 0 : 2 * T * 8;
+  // fused: (max, sum) of each warpgroup [2][T] float2.  pair: each
+  // warpgroup's max [2][T] fp32 and sum [2][T] fp16, then the peer CTA's pushed
+  // (max, sum) [T] float2 at STATS_R
+  static constexpr int STATS = (MODE == kSliced) ? 0 : (MODE == kPair) ? 2 * T * 4 + 2 * T * 2 + T * 8 : 2 * T * 8;
+  static constexpr int STATS_Z = 2 * T * 4, STATS_R = 2 * T * 4 + 2 * T * 2;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_RING = OFF_Q + Q_BYTES;
   static constexpr int OFF_W = OFF_RING + NSLOT * KV_TILE;
@@ -125,14 +130,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(o_full, 1);
     mbar_init(o_empty, kSoftWarps);
     mbar_init(drain, 1);
-    // pair mode: st_ready = warpgroup 1's partials are in, st_used = the final
-    // pair is in (each 4 warps); r_full = the peer's pair has landed (one local
-    // expect_tx + 1 KB of st.async), r_used = the peer has read what this CTA
-    // pushed (the peer's 4 warps of warpgroup 0)
-    mbar_init(st_ready, PAIR ? kSoftWarps / 2 : kSoftWarps);
-    mbar_init(st_used, PAIR ? kSoftWarps / 2 : kSoftWarps);
+    // pair mode: st_ready = both warpgroups' partials are in (8 warps; st_used
+    // is unused); r_full = the peer's pair has landed (one local expect_tx +
+    // 1 KB of st.async), r_used = the peer has read what this CTA pushed (the
+    // peer's 8 softmax warps)
+    mbar_init(st_ready, kSoftWarps);
+    mbar_init(st_used, kSoftWarps);
     mbar_init(r_full, 1);
-    mbar_init(r_used, kSoftWarps / 2);
+    mbar_init(r_used, kSoftWarps);
     *abort_flag = 0;
     *skip_flag = skip ? 1u : 0u;
     fence_mbar_init();
@@ -327,7 +332,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       // pair mode: the peer's R buffer (second half of the stats area) and
       // its barriers, as shared::cluster addresses
-      const uint32_t r_peer = PAIR ? mapa_shared(sbase + C::OFF_STATS + 8u * T, peer) : 0u;
+      const uint32_t r_peer = PAIR ? mapa_shared(sbase + C::OFF_STATS + C::STATS_R, peer) : 0u;
       const uint32_t r_full_peer = PAIR ? mapa_shared(r_full, peer) : 0u;
       const uint32_t r_used_peer = PAIR ? mapa_shared(r_used, peer) : 0u;
       // (max, sum) of two disjoint prototype sets, a before b
@@ -352,7 +357,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(s_empty);
+        // pair mode frees S after the warpgroups have read each other's partials
+        // (that orders every write of the partials after the reads of the last)
+        if (lane == 0 && !PAIR) mbar_arrive(s_empty);
         const bool valid = row < cur.n;
         const int64_t tok = cur.tok0 + row;
         if (MODE == kFused || MODE == kPair) {
@@ -360,36 +367,39 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float z = exp2_shift_sum<C::HALF>(v, c2, m * c2);
           float M, Z, f;
           if (PAIR) {
-            // stats[0..T) = L: warpgroup 1's partial, then the final pair;
-            // stats[T..2T) = R: the peer CTA's combined pair (st.async)
-            float2 fin;
-            if (sw == 1) {
-              stats[row] = make_float2(m, z);
-              __syncwarp();
-              if (lane == 0) mbar_arrive(st_ready);
-              ok = wwait(st_used, li & 1, 0x306);
-              if (!ok) break;
-              fin = stats[row];
-            } else {
-              ok = wwait(st_ready, li & 1, 0x305);
-              if (!ok) break;
-              const float2 loc = combine(make_float2(m, z), stats[row]);
+            // Both warpgroups publish their partial (max, sum) at once; both form
+            // the CTA's pair from the two in warpgroup order, warpgroup 0 pushes
+            // it into the peer CTA (st.async) and both read the peer's push, so
+            // the local and the cluster exchange overlap and every thread of the
+            // pair ends with bitwise the same (max, sum).  The sums travel as
+            // fp16 inside the CTA (a warpgroup's sum lies in [1, 128]).
+            float* lm = reinterpret_cast<float*>(smem + C::OFF_STATS);
+            __half* lz = reinterpret_cast<__half*>(smem + C::OFF_STATS + C::STATS_Z);
+            const float2* rs = reinterpret_cast<const float2*>(smem + C::OFF_STATS + C::STATS_R);
+            lm[sw * T + row] = m;
+            lz[sw * T + row] = __float2half_rn(z);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(st_ready);
+            ok = wwait(st_ready, li & 1, 0x305);
+            if (!ok) break;
+            const float2 loc = combine(make_float2(lm[row], __half2float(lz[row])),
+                                       make_float2(lm[T + row], __half2float(lz[T + row])));
+            __syncwarp();
+            if (lane == 0) mbar_arrive(s_empty);
+            if (sw == 0) {
               if (li > 0) {
                 ok = wwait(r_used, (li - 1) & 1, 0x307);  // the peer has read the last push
                 if (!ok) break;
               }
               if (warp == kSoftWarp0 && lane == 0) mbar_arrive_expect_tx(r_full, 8u * T);
               st_async_f2(r_peer + 8u * row, loc, r_full_peer);
-              ok = wwait(r_full, li & 1, 0x308);
-              if (!ok) break;
-              const float2 oth = stats[T + row];
-              __syncwarp();
-              if (lane == 0) mbar_arrive_relaxed_cluster(r_used_peer);
-              fin = rank == 0 ? combine(loc, oth) : combine(oth, loc);
-              stats[row] = fin;
-              __syncwarp();
-              if (lane == 0) mbar_arrive(st_used);
             }
+            ok = wwait(r_full, li & 1, 0x308);
+            if (!ok) break;
+            const float2 oth = rs[row];
+            __syncwarp();
+            if (lane == 0) mbar_arrive_relaxed_cluster(r_used_peer);
+            const float2 fin = rank == 0 ? combine(loc, oth) : combine(oth, loc);
             M = fin.x;
             Z = fin.y;
             f = ex2((m - M) * c2) / Z;
