@@ -1207,20 +1207,22 @@ struct QCfg {
   static constexpr int KV_TILE = T * D * 2;
   static constexpr int QB = PS * D * 2;
   // K(i) is read by S(i) and, a tile later, by dQ(i); V(i) only by dA(i).  So
-  // K gets three slots and V two: K(i+2) loads once dQ(i-1) is done and V(i+2)
-  // once dA(i) is, each about one tile before it is needed.
-  static constexpr int NK = 3, NV = 2;
+  // K gets four slots and V two: K(i+3) loads once dQ(i-1) is done and V(i+2)
+  // once dA(i) is, a tile or more before they are needed.  (The dsketch slice
+  // lives in TMEM as the A operand of dA, which leaves room for the fourth.)
+  static constexpr int NK = 4, NV = 2;
   static constexpr int NSLOT = NK + NV;
   static constexpr int OFF_Q = 0;
-  static constexpr int OFF_G = QB;
-  static constexpr int OFF_RING = 2 * QB;  // K slots 0..NK-1, then V slots
+  static constexpr int OFF_RING = QB;  // K slots 0..NK-1, then V slots
   static constexpr int OFF_COL = OFF_RING + NSLOT * KV_TILE;  // [2 bufs][lse2 | D][128] fp32
   static constexpr int OFF_BAR = OFF_COL + 2 * 2 * T * 4;
   static constexpr int NBAR = 2 * NSLOT + 16;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // TMEM base, abort flag
   static constexpr int OFF_FLAGS = OFF_MISC + 16;      // per K slot: control bits of the tile it holds
   static constexpr int SMEM = OFF_FLAGS + 4 * NK;
-  static constexpr int S_COL = 0, DA_COL = T, DS_COL = 2 * T, DQ_COL = 3 * T;  // dS: two buffers of T/2
+  // S^T and dA^T fp32; dS (bf16 pairs) and the dsketch slice G (bf16 pairs, the
+  // A operand of dA^T = G V^T) 64 columns each; dQ fp32
+  static constexpr int S_COL = 0, DA_COL = T, DS_COL = 2 * T, G_COL = 2 * T + T / 2, DQ_COL = 3 * T;
   static constexpr int TMEM_COLS = tmem_cols_for(DQ_COL + D);
   static_assert(PS == 128 && TMEM_COLS <= 512 && SMEM <= 232448, "budget");
 };
@@ -1246,7 +1248,7 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
     return;
   }
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t sQ = sbase + C::OFF_Q, sG = sbase + C::OFF_G, sRing = sbase + C::OFF_RING;
+  const uint32_t sQ = sbase + C::OFF_Q, sRing = sbase + C::OFF_RING;
   const uint32_t bar0 = sbase + C::OFF_BAR;
   // slot s < NK holds K tiles, slot NK + j holds V tiles
   auto ring_full = [&](int s) { return bar0 + 8u * s; };
@@ -1274,13 +1276,13 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
     }
     mbar_init(q_full, 1);
     mbar_init(q_empty, 1);
-    mbar_init(g_full, 2);
+    mbar_init(g_full, kSoftWarps);
     mbar_init(g_empty, 1);
     mbar_init(sda_full, 1);
     mbar_init(sda_free, kSoftWarps);
     mbar_init(ds_full, kSoftWarps);
     mbar_init(ds_empty0, 1);
-    mbar_init(ds_empty0 + 8, 1);
+    mbar_init(ds_empty0 + 8, 1);  // unused (one dS buffer)
     mbar_init(dq_empty, kSoftWarps);
     mbar_init(col_full0, 2);
     mbar_init(col_full0 + 8, 2);
@@ -1296,7 +1298,10 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (ntiles > 0) {
+  // Registers: the control warpgroup (warps 0-3: TMA, UMMA issuer, column loaders)
+  // hands registers to the two softmax warpgroups (128 x 136 + 256 x 184 = 384 x 168).
+  if (ntiles > 0 && warp < kSoftWarp0) {
+    setmaxnreg_dec<136>();
     if (warp == 0 && lane == 0) {
       // ---------------------------------------------------------- TMA producer
       tma_prefetch_desc(&tmK);
@@ -1354,7 +1359,7 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
       // built once per operand and stepped by constant offsets.
       constexpr uint32_t idPT = idesc_bf16(128, T, 0, 0);  // [proto x tok], K = d
       constexpr uint32_t idQ = idesc_bf16(128, D, 0, 1);   // [proto x d], K = tokens, A from TMEM
-      const uint64_t dQs = sdesc(sQ, 16, 1024), dGs = sdesc(sG, 16, 1024);
+      const uint64_t dQs = sdesc(sQ, 16, 1024);
       auto step_p = [](int k) { return uint32_t((k >> 2) * (PS * 128) + (k & 3) * 32); };
       auto step_t = [](int k) { return uint32_t((k >> 2) * (T * 128) + (k & 3) * 32); };
       int hc = 0, gc = 0, hp = 0;
@@ -1385,8 +1390,8 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
         for (int k = 0; k < D / 16; ++k)
           umma_ss(tmem + C::S_COL, sdesc_add(dQs, step_p(k)), sdesc_add(dK, step_t(k)), idPT, k > 0 ? 1u : 0u);
 #pragma unroll
-        for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + C::DA_COL, sdesc_add(dGs, step_p(k)), sdesc_add(dV, step_t(k)), idPT, k > 0 ? 1u : 0u);
+        for (int k = 0; k < D / 16; ++k)  // G from TMEM: 8 columns (16 values of d) per step
+          umma_ts(tmem + C::DA_COL, tmem + C::G_COL + 8 * k, sdesc_add(dV, step_t(k)), idPT, k > 0 ? 1u : 0u);
         umma_commit(sda_full);
         umma_commit(ring_empty(sV));                // V read by its only product
         if (fl & kHeadLast) umma_commit(q_empty);   // last S of this head piece
@@ -1412,11 +1417,11 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
         {
           const int sK = k_slot(li);
           const uint64_t dK = sdesc(sRing + sK * C::KV_TILE, T * 128, 1024);  // MN-major: d blocks 16 KB apart
-          const uint32_t dsb = tmem + C::DS_COL + (li & 1) * (T / 2);
+          const uint32_t dsb = tmem + C::DS_COL;
 #pragma unroll
           for (int k = 0; k < T / 16; ++k)
             umma_ts(tmem + C::DQ_COL, dsb + 8 * k, sdesc_add(dK, k * 2048), idQ, (first_of_hp && k == 0) ? 0u : 1u);
-          umma_commit(ds_empty0 + 8 * (li & 1));
+          umma_commit(ds_empty0);
           umma_commit(ring_empty(sK));
         }
         if (fl_cur & kHeadLast) ++hp;
@@ -1425,33 +1430,14 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
       umma_commit(drain);
       mbar_wait_bounded(drain, 0, 200000000ull);
     } else if (warp == 2 || warp == 3) {
-      // ------------------- dsketch slice (fp32 -> bf16, swizzled) and per-token columns
+      // ------------------------------------------------- per-token columns
       const int t64 = threadIdx.x - 64;
       TileWalker cur(a, tb, te, T);
-      int gc = 0;
       bool ok = true;
       auto hw = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
       };
       for (int li = 0; li < ntiles && ok; ++li) {
-        if (cur.seg_first) {
-          if (gc > 0) ok = hw(g_empty, (gc - 1) & 1, 0xE01);
-          if (!ok) break;
-          const float* src = dsk + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D;
-          constexpr int CHUNKS = PS * D / 8;
-          for (int c = t64; c < CHUNKS; c += 64) {
-            const int p = c / (D / 8), dd = (c % (D / 8)) * 8;
-            const float4 x = *reinterpret_cast<const float4*>(src + int64_t(p) * D + dd);
-            const float4 y = *reinterpret_cast<const float4*>(src + int64_t(p) * D + dd + 4);
-            const int dh = dd >> 6, chunk = (dd & 63) >> 3;
-            *reinterpret_cast<uint4*>(smem + C::OFF_G + dh * PS * 128 + p * 128 + ((chunk ^ (p & 7)) << 4)) =
-                make_uint4(pack_bf16(x.x, x.y), pack_bf16(x.z, x.w), pack_bf16(y.x, y.y), pack_bf16(y.z, y.w));
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(g_full);
-          ++gc;
-        }
         if (!TW) {
           const int buf = li & 1;
           if (li >= 2) ok = hw(col_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xE02);
@@ -1468,13 +1454,44 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
         }
         cur.next();
       }
-    } else if (warp >= kSoftWarp0) {
+    }
+  } else if (ntiles > 0) {
+    setmaxnreg_inc<184>();
+    {
       // ------------------------------------------------ dS + dQ epilogue
       const int sw = (warp - kSoftWarp0) >> 2, q = warp & 3;
       const uint32_t lane_off = uint32_t(32 * q) << 16;
       const float c2 = a.scale * 1.4426950408889634f;
       TileWalker cur(a, tb, te, T);
       bool ok = true;
+      int gc = 0;
+      // The dsketch slice of user b, head h into TMEM as bf16 pairs (the A operand of
+      // dA^T = G V^T): this thread's prototype row, warpgroup sw's half of the d columns.
+      // Written once the last dA of the previous segment is done (g_empty).
+      auto put_g = [&](int b, int h) -> bool {
+        if (gc > 0 && !__all_sync(0xffffffffu, mbar_wait(g_empty, (gc - 1) & 1, abort_flag, a.ws, 0xF06)))
+          return false;
+        const float4* src = reinterpret_cast<const float4*>(
+            dsk + ((int64_t(b) * a.H + h) * a.P + p0 + 32 * q + lane) * D + (D / 2) * sw);
+#pragma unroll
+        for (int half = 0; half < D / 64; ++half) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 x = src[8 * half + j];
+            pk[2 * j] = pack_bf16(x.x, x.y);
+            pk[2 * j + 1] = pack_bf16(x.z, x.w);
+          }
+          tmem_st16(tmem + lane_off + C::G_COL + (D / 4) * sw + 16 * half, pk);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(g_full);
+        ++gc;
+        return true;
+      };
+      ok = put_g(cur.b, cur.h);
       auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
       };
@@ -1490,8 +1507,6 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
           ok = wwait(col_full0 + 8 * buf, (li >> 1) & 1, 0xF01);
         }
         if (ok) ok = wwait(sda_full, li & 1, 0xF02);
-        // this tile's dS buffer was last read by dQ(i-2)
-        if (ok && li > 1) ok = wwait(ds_empty0 + 8 * buf, ((li >> 1) + 1) & 1, 0xF04);
         if (!ok) break;
         tc_fence_after();
         const float* cl = cols + buf * 2 * T;
@@ -1503,6 +1518,15 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
         tmem_ld_wait();
         tc_fence_before();
         __syncwarp();
+        // the next tile opens a new (user, head) segment: its dsketch slice goes in
+        // before S and dA of that tile are issued (they wait for sda_free and g_full)
+        if (li + 1 < ntiles && cur.seg_last) {
+          const TileRef nx = locate_tile(cur.t + 1, cur.tph, a.prefix, a.cu, a.B, T);
+          if (!put_g(nx.b, nx.h)) {
+            ok = false;
+            break;
+          }
+        }
         if (lane == 0) mbar_arrive(sda_free);  // the next tile's S and dA may now be written
         if (TW) {
           // per-row shift and D; columns past the tile's tokens weigh zero
@@ -1517,8 +1541,14 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
               const float a1 = col + 2 * j + 1 < cur.n ? ex2(fmaf(sv[jj + 1], c2, -l2r)) : 0.f;
               pk[j] = pack_bf16(a0 * (dv[jj] - dr), a1 * (dv[jj + 1] - dr));
             }
-            tmem_st16(tmem + lane_off + C::DS_COL + buf * (T / 2) + col / 2, pk);
+            // dS(i) overwrites dS(i-1): dQ(i-1) must have read it
+            if (c == 0 && li > 0 && !wwait(ds_empty0, (li - 1) & 1, 0xF04)) {
+              ok = false;
+              break;
+            }
+            tmem_st16(tmem + lane_off + C::DS_COL + col / 2, pk);
           }
+          if (!ok) break;
         }
         // per-token values as 16-byte broadcasts: one shared-memory wavefront per 4 tokens
         const float4* cl4 = reinterpret_cast<const float4*>(cl);
@@ -1536,8 +1566,13 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
             pk[2 * j4] = pack_bf16(a0 * (dv[jj] - d4.x), a1 * (dv[jj + 1] - d4.y));
             pk[2 * j4 + 1] = pack_bf16(a2 * (dv[jj + 2] - d4.z), a3 * (dv[jj + 3] - d4.w));
           }
-          tmem_st16(tmem + lane_off + C::DS_COL + buf * (T / 2) + col / 2, pk);
+          if (c == 0 && li > 0 && !wwait(ds_empty0, (li - 1) & 1, 0xF04)) {
+            ok = false;
+            break;
+          }
+          tmem_st16(tmem + lane_off + C::DS_COL + col / 2, pk);
         }
+        if (!ok) break;
         tmem_st_wait();
         tc_fence_before();
         __syncwarp();
@@ -1551,7 +1586,7 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
         int nn, hn, qkn;
         cur.peek_next(t0n, nn, hn, qkn);
         if (!more || qkn != cur.qk) {
-          ok = wwait(ds_empty0 + 8 * buf, (li >> 1) & 1, 0xF05);
+          ok = wwait(ds_empty0, li & 1, 0xF05);
           if (!ok) break;
           tc_fence_after();
           float* dst = dq_block_dst(a, wk, W, total, cur, p0, D);
