@@ -18,6 +18,9 @@ worker accumulates its ~42K tokens per head in TMEM (fp32, about 2600 UMMA
 steps) and the two splits group the tokens differently; the sums agree to a
 few 1e-3 of max|dQ| (2.2e-3 measured), so the check uses 1e-2 -- a lost or
 doubled worker piece would move dQ by about 1/sqrt(38 workers) ~ 16 %.
+
+Device memory: K and V take 26 GB each and every backward allocates dK and dV of
+the same size, so the tests hold up to ~140 GB (a GB300 has 288 GB).
 """
 import numpy as np
 import pytest
