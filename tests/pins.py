@@ -481,6 +481,30 @@ def pin_tw_bruteforce(fwd_tw, bwd_tw=None, fwd=None, bwd=None):
                     assert abs(O[b, h, j, c] - float(ref)) <= 1e-12 * max(1.0, abs(float(ref))), (b, h, j, c)
 
 
+def pin_tw_bruteforce_lse(fwd_tw, bwd_tw=None, fwd=None, bwd=None):
+    """50-digit plain loops of lse_tok[b, h, j] = log sum_i exp(S[j, i]) over
+    user b's tokens (no stabilising shift), and -inf for a user with none."""
+    import mpmath as mp
+
+    mp.mp.dps = 50
+    lens = [4, 0, 1, 3]
+    K, V, cu, Q, _ = _rand_problem(58, lens, H=2, P=3, d=3, q_std=2.0)
+    scale = 1.1
+    _, lse = fwd_tw(K, V, cu, Q, scale, with_lse=True)
+    assert lse.shape == (len(lens), 2, 3), f"lse_tok shape {lse.shape}"
+    for b in range(len(lens)):
+        t0, t1 = int(cu[b]), int(cu[b + 1])
+        for h in range(2):
+            for j in range(3):
+                if t1 == t0:
+                    assert lse[b, h, j] == -np.inf, (b, h, j)
+                    continue
+                z = mp.fsum(mp.exp(mp.mpf(scale) * mp.fsum(mp.mpf(Q[h, j, c]) * mp.mpf(K[i, h, c])
+                                                         for c in range(3))) for i in range(t0, t1))
+                ref = float(mp.log(z))
+                assert abs(lse[b, h, j] - ref) <= 1e-12 * max(1.0, abs(ref)), (b, h, j, lse[b, h, j], ref)
+
+
 def pin_tw_rows_sum_to_one(fwd_tw, bwd_tw=None, fwd=None, bwd=None):
     """V = 1: every sketch entry of a non-empty user is 1 (sum_i A[j, i] = 1)."""
     lens = [4, 0, 9]
@@ -544,4 +568,4 @@ def pin_tw_fd_fp64(fwd_tw, bwd_tw, fwd=None, bwd=None):
             assert abs(grad[idx] - ref) <= 1e-6 * max(1.0, abs(ref)), f"d{name}{idx}"
 
 
-TW_PINS = [pin_tw_bruteforce, pin_tw_rows_sum_to_one, pin_tw_closed_forms, pin_tw_token_order, pin_tw_fd_fp64]
+TW_PINS = [pin_tw_bruteforce, pin_tw_bruteforce_lse, pin_tw_rows_sum_to_one, pin_tw_closed_forms, pin_tw_token_order, pin_tw_fd_fp64]

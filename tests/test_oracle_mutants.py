@@ -167,11 +167,31 @@ def test_key_projection_mutant_is_caught(name):
 
 
 # ------------------------- token-wise ("vanilla") normalisation (Sec. 5.1)
-def _tw_variant(proto_axis=False, drop_d=False, dv_from_g_t=False):
+def _tw_lse_variant(lse_axis=1, keep_max=True):
+    """lse_tok computed with the reduction over the wrong axis (axis 0, the
+    prototypes) or with the subtracted maximum not added back."""
+    def lse_tok(S):
+        m = S.max(axis=lse_axis, keepdims=True)
+        r = np.log(np.exp(S - m).sum(axis=lse_axis, keepdims=True)) + (m if keep_max else 0.0)
+        return np.broadcast_to(r, S.shape)[:, 0]
+    return lse_tok
+
+
+def _tw_variant(proto_axis=False, drop_d=False, dv_from_g_t=False, lse_fn=None):
     def fwd(K, V, cu, Q, scale, with_lse=False):
         if proto_axis:
             return so.sa_forward(K, V, cu, Q, scale, with_lse=with_lse)
-        return so.sa_forward_tokenwise(K, V, cu, Q, scale, with_lse=with_lse)
+        if lse_fn is None or not with_lse:
+            return so.sa_forward_tokenwise(K, V, cu, Q, scale, with_lse=with_lse)
+        O = so.sa_forward_tokenwise(K, V, cu, Q, scale)
+        Qd = np.asarray(Q, float)
+        lse = np.full(O.shape[:3], -np.inf)
+        for b, (t0, t1) in enumerate(so._user_slices(cu)):
+            if t1 == t0:
+                continue
+            for h in range(Qd.shape[0]):
+                lse[b, h] = lse_fn(scale * (Qd[h] @ np.asarray(K, float)[t0:t1, h].T))
+        return O, lse
 
     def bwd(K, V, cu, Q, scale, dO):
         K = np.asarray(K, float); V = np.asarray(V, float); Q = np.asarray(Q, float); dO = np.asarray(dO, float)
@@ -197,6 +217,8 @@ TW_MUTANTS = {
     "normalised over prototypes": _tw_variant(proto_axis=True),
     "dS without the row term": _tw_variant(drop_d=True),
     "dV with prototypes reversed": _tw_variant(dv_from_g_t=True),
+    "lse_tok reduced over the prototypes": _tw_variant(lse_fn=_tw_lse_variant(lse_axis=0)),
+    "lse_tok without its maximum": _tw_variant(lse_fn=_tw_lse_variant(keep_max=False)),
 }
 
 
