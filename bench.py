@@ -23,6 +23,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -35,7 +36,6 @@ from paper_2609_08443_gb300 import workloads as wl  # noqa: E402
 
 METRIC = "SA sketched tokens/sec fwd and fwd+bwd at 100K/user; % of roofline"
 CONFIG_ID = 4
-E2E_USERS = 16
 
 
 def peaks():
@@ -43,8 +43,10 @@ def peaks():
     if os.path.exists(p):
         d = json.load(open(p))
         return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
-                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]), "source": "measured"}
-    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                "sm_max_mhz": d.get("sm_max_mhz", 2070.0), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0,
+            "source": "fallback"}
 
 
 def workload_config(spec, lens):
@@ -66,11 +68,11 @@ class Clocks:
     def __init__(self, gpu_index):
         self.gpu = gpu_index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_bench_{os.getpid()}.csv")
+        fd, self.path = tempfile.mkstemp(prefix="sa_bench_clocks_", suffix=".csv")
+        os.close(fd)
 
     def __enter__(self):
         try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
                                           "--format=csv,noheader,nounits", "-lms", "200"],
@@ -87,13 +89,18 @@ class Clocks:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
             self.fh.close()
+        self.lines = open(self.path).read().splitlines() if os.path.exists(self.path) else []
+        try:
+            os.remove(self.path)
+        except OSError:
+            pass
 
     def summary(self):
-        if self.proc is None or not os.path.exists(self.path):
+        if self.proc is None or not self.lines:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         sm, smax, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in open(self.path):
+        for line in self.lines:
             f = [x.strip() for x in line.split(",")]
             if len(f) < 9:
                 continue
@@ -293,11 +300,18 @@ def run_ours(args, spec, lens):
     fwd_name = binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
     r_bwd = roof(bw, bwd_k_ms, bwd_k_n, bwd_name, args.steps)
     r_fwd = roof(fw, fwd_k_ms, fwd_k_n, fwd_name, args.steps)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    exp_ps = rf.exp_peak_per_s(sms, pk["sm_max_mhz"])
     step_w = rf.step_work(tokens, B, H, P, d, eb)
-    t_roof = rf.roofline_time(step_w, peak_t, pk["hbm_gbs"])
+    t_roof = rf.roofline_time(step_w, peak_t, pk["hbm_gbs"], exp_ps)
+    t_roof_fwd = rf.roofline_time(fw, peak_t, pk["hbm_gbs"], exp_ps)
 
     tw = tokenwise_leg(args, spec, data, dev, pk) if rank == 0 else None
-    e2e = e2e_run(args, spec, dev) if rank == 0 else None
+    e2e = e2e_run(args, spec, data, (dK, dV), dev) if rank == 0 else None
+    # the other workloads, after the 100K batch's buffers are released
+    del data, K, V, Q, cu, dS, sketch, lse, dK, dV, dQ, ws
+    torch.cuda.empty_cache()
+    others = {f"config{i}": config_leg(i, args, dev, pk, exp_ps) for i in (1, 2, 3, 5)} if rank == 0 else None
     cpu = oracle_sample(spec, budget_s=15.0) if (rank == 0 and world == 1) else None
 
     if rank == 0:
@@ -306,15 +320,97 @@ def run_ours(args, spec, lens):
                 "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
                 "config": workload_config(spec, lens),
                 "fwd": {"value": tokens * world / (fwd_ms / 1e3), "unit": "tokens/s", "ms_per_call": fwd_ms,
-                        "roofline_frac": (rf.roofline_time(fw, peak_t, pk["hbm_gbs"])["time"] * 1e3) / fwd_ms},
+                        "roofline_bound": t_roof_fwd["bound"], "roofline_ms": t_roof_fwd["time"] * 1e3,
+                        "roofline_frac": (t_roof_fwd["time"] * 1e3) / fwd_ms},
                 "step_roofline": {"bound": t_roof["bound"], "ms": t_roof["time"] * 1e3,
-                                  "frac": t_roof["time"] * 1e3 / ms_per_step},
+                                  "frac": t_roof["time"] * 1e3 / ms_per_step,
+                                  "terms_ms": {k: t_roof[k] * 1e3 for k in ("tensor", "hbm", "mufu")}},
+                "mufu_peak": {"ex2_per_s": exp_ps, "per_sm_clk": rf.EX2_PER_SM_CLK, "sms": sms,
+                              "sm_mhz": pk["sm_max_mhz"], "source": "ex2.approx throughput probe (measured)"},
                 "roofline": r_bwd, "roofline_fwd": r_fwd,
                 "cpu_baseline": cpu, "e2e": e2e, "clocks": clk.summary(), "gpu_launches": int(launches),
-                "kernels": {"fwd": fwd_name, "bwd": bwd_name}, "kernel_ms": per_kernel, "tokenwise": tw}
+                "kernels": {"fwd": fwd_name, "bwd": bwd_name}, "kernel_ms": per_kernel, "tokenwise": tw,
+                "workloads": others}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def config_leg(cfg, args, dev, pk, exp_ps):
+    """One of the other evaluation workloads at full size through the C ABI:
+    the forward alone and, where the workload trains, forward (saving lse) +
+    backward, each timed over K calls with CUDA events after warm-up, against
+    its roofline (slowest of tensor FLOPs, HBM bytes and exp2 at their peaks).
+    Reported beside the headline, not part of it."""
+    import torch
+
+    from paper_2609_08443_gb300 import binding
+
+    spec = wl.config(cfg)
+    lens = wl.lengths(spec)
+    data = wl.make_device(spec, dev)
+    K, V, Q, cu, dS = data["K"], data["V"], data["Q"], data["cu_seqlens"], data["dsketch"]
+    B = int(lens.size)
+    N, H, d = K.shape
+    P = Q.shape[1]
+    tokens = int(lens.sum())
+    code = binding.SA_BF16 if K.dtype == torch.bfloat16 else binding.SA_F32
+    eb = K.element_size()
+    sketch = torch.empty((B, H, P, d), dtype=torch.float32, device=dev)
+    lse = torch.empty((N, H), dtype=torch.float32, device=dev)
+    ws = torch.empty(binding.sa_workspace_size(B, N, H, P, d, code, int(spec.bwd)), dtype=torch.uint8, device=dev)
+    outs = (torch.empty_like(K), torch.empty_like(V), torch.empty((H, P, d), dtype=torch.float32, device=dev))
+    stream = torch.cuda.current_stream(dev)
+    # small workloads: more calls per timing so the events cover well over a millisecond
+    reps = max(args.steps, 20)
+
+    def timed(fn):
+        for _ in range(args.warmup):
+            fn()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / reps
+
+    def fwd():
+        binding.sa_sketch_fwd(K, V, cu, Q, spec.scale, out=sketch, lse_out=lse, ws=ws)
+
+    def step():
+        fwd()
+        binding.sa_sketch_bwd(K, V, cu, Q, dS, spec.scale, lse=lse, outs=outs, ws=ws)
+
+    # fp32 inputs run on the CUDA cores: their compute term is the FP32 FMA rate
+    # (128 lanes x 2 FLOP per SM and clock), not the bf16 tensor peak
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak_c = pk["bf16_tflops"] if code == binding.SA_BF16 else sms * 128 * 2 * pk["sm_max_mhz"] * 1e6 / 1e12
+    cname = "tensor" if code == binding.SA_BF16 else "fp32_fma"
+
+    def entry(ms, work):
+        r = rf.roofline_time(work, peak_c, pk["hbm_gbs"], exp_ps)
+        bound = cname if r["bound"] == "tensor" else r["bound"]
+        return {"ms": ms, "tokens_per_s": tokens / (ms / 1e3), "roofline_bound": bound,
+                "roofline_ms": r["time"] * 1e3, "roofline_frac": r["time"] * 1e3 / ms,
+                "terms_ms": {cname: r["tensor"] * 1e3, "hbm": r["hbm"] * 1e3, "mufu": r["mufu"] * 1e3}}
+
+    out = {"workload": spec.name, "users": B, "tokens": tokens, "heads": H, "d": d, "prototypes": P,
+           "dtype": "bf16" if code == binding.SA_BF16 else "f32",
+           "kernels": {"fwd": binding.sa_main_kernel_name(P, d, code, False)},
+           "tile_fill": tokens / (128.0 * int(np.sum((lens + 127) // 128))),
+           "timing": f"CUDA events over {reps} calls after {args.warmup} warm-up calls; peaks: bf16 burst, HBM copy, "
+                     "MUFU ex2 (measured)"}
+    out["fwd"] = entry(timed(fwd), rf.fwd_work(tokens, B, H, P, d, eb, lse=True))
+    if spec.bwd:
+        out["kernels"]["bwd"] = binding.sa_main_kernel_name(P, d, code, True)
+        out["fwd_bwd"] = entry(timed(step), rf.step_work(tokens, B, H, P, d, eb))
+    if binding.sa_get_device_error(ws) != 0:
+        raise RuntimeError(f"device-side error in workload {cfg}")
+    del data, K, V, ws, outs
+    torch.cuda.empty_cache()
+    return out
 
 
 def tokenwise_leg(args, spec, data, dev, pk):
@@ -389,37 +485,96 @@ def traffic_for(kernel_name):
     return ent.get("bytes_per_call") if ent.get("source_hash") == build.source_hash() else None
 
 
-def e2e_run(args, spec, dev):
+def _meminfo_available():
+    try:
+        for line in open("/proc/meminfo"):
+            if line.startswith("MemAvailable:"):
+                return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return None
+
+
+def copy_ceiling(h_src, h_dst, d_buf, dev, nbytes):
+    """Plain page-locked copies of ``nbytes``: host-to-device alone,
+    device-to-host alone, and both at once on two streams (GB/s, CUDA events)."""
+    import torch
+
+    n = nbytes // h_src.element_size()
+    hs, hd, db = h_src.view(-1)[:n], h_dst.view(-1)[:n], d_buf.view(-1)
+    dbi, dbo = db[:n], db[n:2 * n]
+    s1, s2 = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+
+    def run(h2d, d2h):
+        torch.cuda.synchronize(dev)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ev[0].record(s1)
+        s2.wait_event(ev[0])
+        if h2d:
+            with torch.cuda.stream(s1):
+                dbi.copy_(hs, non_blocking=True)
+        if d2h:
+            with torch.cuda.stream(s2):
+                hd.copy_(dbo, non_blocking=True)
+        ev[1].record(s1)
+        ev[2].record(s2)
+        torch.cuda.synchronize(dev)
+        ms = max(ev[0].elapsed_time(ev[1]), ev[0].elapsed_time(ev[2]))
+        return (int(h2d) + int(d2h)) * nbytes / (ms / 1e3) / 1e9
+
+    run(True, True)  # warm
+    return {"h2d_gbs": max(run(True, False) for _ in range(3)), "d2h_gbs": max(run(False, True) for _ in range(3)),
+            "both_gbs": max(run(True, True) for _ in range(3)), "bytes_each": int(nbytes),
+            "how": "torch copy_ between page-locked host and device memory, CUDA events, best of 3"}
+
+
+def e2e_run(args, spec, data, dkdv, dev):
     """Same metric through the public API with host buffers: every step hands the
     library page-locked host arrays (K, V, Q, dsketch) and gets the host arrays
     (sketch, dK, dV, dQ) back, through sa_sketch_step_host, which copies chunks of
     users in and out on its own streams while the step runs on the previous
-    chunk.  Wall clock from the call to the synchronised results."""
+    chunk.  Wall clock from the call to the synchronised results, every user of
+    the workload unless the host lacks the page-locked memory for them."""
     import torch
 
     from paper_2609_08443_gb300 import binding
 
-    sub = wl.sub_spec(spec, list(range(E2E_USERS)))
-    lens = wl.lengths(sub)
-    d_in = wl.make_device(sub, dev)
-    h = {k: v.to("cpu").pin_memory() for k, v in d_in.items() if hasattr(v, "pin_memory")}
-    del d_in
-    B, H, P, d = sub.B, sub.H, sub.P, sub.d
-    N = int(lens.sum())
-    outs = (torch.empty((B, H, P, d), dtype=torch.float32).pin_memory(),
-            torch.empty((N, H, d), dtype=torch.bfloat16).pin_memory(),
-            torch.empty((N, H, d), dtype=torch.bfloat16).pin_memory(),
-            torch.empty((H, P, d), dtype=torch.float32).pin_memory())
-    cu = h["cu_seqlens"]
+    lens = wl.lengths(spec)
+    B_all, H, P, d = spec.B, spec.H, spec.P, spec.d
+
+    def pinned_need(b):
+        # torch's page-locked allocator rounds each block up to a power of two
+        n = int(lens[:b].sum())
+        sizes = [n * H * d * 2] * 4 + [b * H * P * d * 4] * 2
+        return sum(1 << (max(s, 1) - 1).bit_length() for s in sizes)
+
+    avail = _meminfo_available()
+    B = B_all
+    while avail is not None and B > 1 and pinned_need(B) > 0.85 * avail:
+        B -= 1
+    N = int(lens[:B].sum())
+    cu = torch.from_numpy(wl.cu_seqlens(lens[:B]))
+    pin = dict(dtype=torch.bfloat16, pin_memory=True)
+    h = {"K": torch.empty((N, H, d), **pin), "V": torch.empty((N, H, d), **pin),
+         "Q": torch.empty((H, P, d), **pin), "dsketch": torch.empty((B, H, P, d), dtype=torch.float32,
+                                                                     pin_memory=True),
+         "cu_seqlens": cu.pin_memory()}
+    for k in ("K", "V"):
+        h[k].copy_(data[k][:N])
+    h["Q"].copy_(data["Q"])
+    h["dsketch"].copy_(data["dsketch"][:B])
+    outs = (torch.empty((B, H, P, d), dtype=torch.float32, pin_memory=True), torch.empty((N, H, d), **pin),
+            torch.empty((N, H, d), **pin), torch.empty((H, P, d), dtype=torch.float32, pin_memory=True))
+    ceiling = copy_ceiling(h["K"], outs[1], dkdv[0], dev, min(4 << 30, h["K"].numel() * 2 // 2))
     lib = binding.load()
-    ws = torch.empty(lib.sa_step_host_workspace_size(cu.data_ptr(), B, H, P, d, binding.SA_BF16, 0),
+    ws = torch.empty(lib.sa_step_host_workspace_size(h["cu_seqlens"].data_ptr(), B, H, P, d, binding.SA_BF16, 0),
                      dtype=torch.uint8, device=dev)
     h2d = sum(h[k].numel() * h[k].element_size() for k in ("K", "V", "Q", "dsketch", "cu_seqlens"))
     d2h = sum(o.numel() * o.element_size() for o in outs)
 
     def step():
-        binding.sa_sketch_step_host(h["K"], h["V"], cu, h["Q"], h["dsketch"], sub.scale, outs=outs, device=dev,
-                                    ws=ws)
+        binding.sa_sketch_step_host(h["K"], h["V"], h["cu_seqlens"], h["Q"], h["dsketch"], spec.scale, outs=outs,
+                                    device=dev, ws=ws)
 
     for _ in range(3):
         step()
@@ -431,12 +586,16 @@ def e2e_run(args, spec, dev):
         t0 = time.perf_counter()
         step()
         times.append(time.perf_counter() - t0)
-    dt = statistics.median(times)
-    return {"value": N / dt, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-            "sample": f"{E2E_USERS} of the 128 users (same shapes), page-locked host arrays in and out through "
+    mean = sum(times) / len(times)
+    med = statistics.median(times)
+    return {"value": N / mean, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "sample": f"{B} of the {B_all} users (same shapes), page-locked host arrays in and out through "
                       "sa_sketch_step_host (chunks of 262144 tokens, copies overlapped with the step), wall clock, "
-                      f"median of {n} steps",
-            "ms_per_step": dt * 1e3, "ms_per_step_all": [t * 1e3 for t in times]}
+                      f"mean of {n} steps" + ("" if B == B_all else
+                                              f"; host MemAvailable {avail / 2**30:.0f} GiB limits the users"),
+            "ms_per_step": mean * 1e3, "ms_per_step_median": med * 1e3, "value_median": N / med,
+            "ms_per_step_all": [t * 1e3 for t in times],
+            "copy_gbs": (h2d + d2h) / mean / 1e9, "copy_ceiling": ceiling}
 
 
 def main():

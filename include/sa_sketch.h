@@ -75,8 +75,10 @@ size_t sa_workspace_size(int B, int64_t N, int H, int P, int d, sa_dtype dt, int
 /* Forward: sketch[b,h] = softmax_proto(scale * Q[h] K_b[:,h]^T) V_b[:,h]
  * (Sec. 3.1).  `lse` may be NULL; when given it receives, per token and head,
  * log sum_j exp(S[j,i]) (the softmax statistic FlashSA keeps, Sec. 4.4) so the
- * backward can skip recomputing it.  `scale` is normally 1/sqrt(d); a negative
- * scale is valid and runs on the CUDA-core kernels. */
+ * backward can skip recomputing it.  `scale` is normally 1/sqrt(d); any finite
+ * scale is valid.  A negative one runs on the same tensor-core kernels: the
+ * call negates a copy of Q in the workspace (scale Q K^T = (-scale)(-Q) K^T,
+ * exactly), and the backward negates dQ back. */
 sa_status sa_sketch_fwd(const void* K, const void* V, const int32_t* cu_seqlens, int B,
                         int64_t N, const void* Q, int H, int P, int d, float scale,
                         sa_dtype dt, float* sketch, float* lse, void* workspace,
@@ -147,8 +149,11 @@ sa_status sa_sketch_bwd_x(const void* X, const int32_t* cu_seqlens, int B, int64
  *     sketch[b, h] = A V_b                          (P x d)
  *     lse_tok      : [B, H, P] fp32, log sum_i exp(S[j, i]) per user, head and
  *                    prototype (-inf for a user with L_b = 0, whose sketch is 0)
- * `lse_tok` may be NULL.  Shared prototypes Q [H, P, d] only.  CUDA-core
- * kernels (fp32 arithmetic) for both dtypes.  The workspace must hold
+ * `lse_tok` may be NULL.  Shared prototypes Q [H, P, d] only.  Tensor cores
+ * (tcgen05, fp32 accumulation) serve bf16 with d in {64, 128} and P a multiple
+ * of 128 up to 2048, for any nonzero scale (a negative one is folded into a
+ * negated copy of Q as in sa_sketch_fwd); other shapes, fp32 inputs and a zero
+ * scale run on CUDA-core kernels (fp32 arithmetic).  The workspace must hold
  * sa_workspace_size_tokenwise() bytes; everything else (layouts, ownership,
  * errors, determinism) as in sa_sketch_fwd. */
 size_t sa_workspace_size_tokenwise(int B, int64_t N, int H, int P, int d, sa_dtype dt, int bwd);
@@ -210,18 +215,36 @@ sa_status sa_sketch_step_host(const void* K, const void* V, const int32_t* cu_se
  * device memory on every GPU where it is loaded, until the process exits.
  *   - Returns SA_ERR_WORKSPACE, before launching anything, when the call would
  *     need more scratch than that (large N, B, P or d); use sa_sketch_fwd then.
- *   - It allocates nothing.  The first call on a device looks up the array's
- *     device address (cudaGetSymbolAddress, with that device current) and
- *     caches it; make that first call before any stream capture.
+ *   - It allocates nothing itself.  The array belongs to the current device
+ *     (cudaGetDevice), not to the device of `stream` or of the tensors: make
+ *     the device that owns the stream and all buffers current before calling.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current) and caches it with the
+ *     device's context (a reset context is looked up again).  Under CUDA's
+ *     default lazy module loading that first call is also when the driver
+ *     commits the array's 32 MiB, so it can fail with SA_ERR_CUDA if the
+ *     device is out of memory: make one warm-up call at set-up, before the
+ *     memory budget is fully used and before any stream capture.
  *   - All calls share the one array: two calls whose work overlaps on the GPU
  *     (different streams, or different host threads) race and may corrupt each
- *     other's results; serialise them.  Each call rewrites everything it reads. */
+ *     other's results; serialise them.  Each call rewrites everything it
+ *     reads, including the error word, so a call after a failed one starts
+ *     clean.
+ *   - Errors only the device can see (bad cu_seqlens contents, a pipeline wait
+ *     that gave up) make the call's kernels skip their work and are reported
+ *     by sa_noalloc_get_device_error(), not by the return value. */
 sa_status sa_sketch_fwd_noalloc(const void* K, const void* V, const int32_t* cu_seqlens, int B,
                                 int64_t N, const void* Q, int H, int P, int d, float scale,
                                 sa_dtype dt, float* sketch, float* lse, void* stream);
 
 /* Size in bytes of the fixed scratch array used by sa_sketch_fwd_noalloc. */
 size_t sa_noalloc_scratch_bytes(void);
+
+/* Synchronises `stream` and returns the device-detected status of the last
+ * sa_sketch_fwd_noalloc call on the current device (SA_OK, SA_ERR_BAD_SEQLENS
+ * or SA_ERR_TIMEOUT), or SA_ERR_CUDA if the stream reports an error.  The
+ * counterpart of sa_get_device_error() for callers that hold no workspace. */
+sa_status sa_noalloc_get_device_error(void* stream);
 
 /* Synchronises `stream` and returns the device-detected status of the last call
  * that used this workspace (SA_OK, SA_ERR_BAD_SEQLENS or SA_ERR_TIMEOUT), or
@@ -255,6 +278,16 @@ sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches)
 
 /* Number of kernels this library has launched in this process. */
 uint64_t sa_launch_count(void);
+
+/* Time limit, in nanoseconds, of every bounded wait inside the tensor-core
+ * kernels, for calls enqueued after this one (0 restores the default of 2 s;
+ * at most 60 s, else SA_ERR_INVALID_ARG).  A correct pipeline never waits
+ * anywhere near 2 s; a lower limit exists so that tests can make a wait run
+ * out on purpose and check the recovery: the call's kernels stop, drain their
+ * copies and tensor-core work still in flight, release their tensor memory,
+ * and sa_get_device_error() reports SA_ERR_TIMEOUT.  The limit is copied into
+ * each call's workspace when the call is enqueued. */
+sa_status sa_set_wait_limit_ns(uint64_t ns);
 
 /* Kernel selection for all later calls in this process: 0 (default) lets each
  * call pick the tensor-core kernels where its shape is supported, 1 forces the

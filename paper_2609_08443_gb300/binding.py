@@ -76,6 +76,10 @@ def load() -> ctypes.CDLL:
     lib.sa_sketch_fwd_noalloc.restype = i32
     lib.sa_noalloc_scratch_bytes.argtypes = []
     lib.sa_noalloc_scratch_bytes.restype = sz
+    lib.sa_noalloc_get_device_error.argtypes = [vp]
+    lib.sa_noalloc_get_device_error.restype = i32
+    lib.sa_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
+    lib.sa_set_wait_limit_ns.restype = i32
     lib.sa_workspace_size_tokenwise.argtypes = [i32, i64, i32, i32, i32, i32, i32]
     lib.sa_workspace_size_tokenwise.restype = sz
     lib.sa_sketch_fwd_tokenwise.argtypes = lib.sa_sketch_fwd.argtypes
@@ -277,10 +281,26 @@ def sa_sketch_fwd_noalloc(K: torch.Tensor, V: torch.Tensor, cu_seqlens: torch.Te
     B = cu_seqlens.numel() - 1
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
     sketch = out if out is not None else torch.empty((B, H, P, d), dtype=torch.float32, device=K.device)
-    st = lib.sa_sketch_fwd_noalloc(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale, _dt(K),
-                                   _ptr(sketch), _ptr(lse_out), _stream(K.device))
+    # the library uses the fixed array of the CURRENT device: make K's device current
+    with torch.cuda.device(K.device):
+        st = lib.sa_sketch_fwd_noalloc(_ptr(K), _ptr(V), _ptr(cu_seqlens), B, N, _ptr(Q), H, P, d, scale,
+                                       _dt(K), _ptr(sketch), _ptr(lse_out), _stream(K.device))
     _check(st, "sa_sketch_fwd_noalloc")
     return sketch
+
+
+def sa_noalloc_get_device_error(device=None) -> int:
+    """Device-detected status of the last sa_sketch_fwd_noalloc call on
+    ``device`` (synchronises its current stream)."""
+    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    with torch.cuda.device(device):
+        return int(load().sa_noalloc_get_device_error(_stream(device)))
+
+
+def sa_set_wait_limit_ns(ns: int) -> None:
+    """Limit of the kernels' bounded pipeline waits for later calls (0 = the
+    default 2 s); a test hook for the timeout path."""
+    _check(load().sa_set_wait_limit_ns(int(ns)), "sa_set_wait_limit_ns")
 
 
 def _validate_x(X, cu, Q, Wk):

@@ -19,6 +19,9 @@ std::atomic<int> g_path{0};  // 0 = choose per shape, 1 = CUDA cores only, 2 = l
 
 std::atomic<uint64_t> g_launches{0};
 
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;  // 2 s
+std::atomic<uint64_t> g_wait_ns{kDefaultWaitNs};
+
 int device_sms() {
   static int cache[64] = {0};
   int dev = 0;
@@ -94,7 +97,9 @@ bool shape_ok(int B, int64_t N, int H, int P, int d, sa_dtype dt) {
 
 // allow_tc = false keeps every kernel on the CUDA cores: the tensor-core
 // kernels take the softmax maximum on the raw scores, which is the maximum of
-// the scaled scores only for scale >= 0.
+// the scaled scores only for scale >= 0.  With shared prototypes a negative
+// scale is folded into them instead (fold_negative_scale), so only per-user
+// queries with a negative scale need the CUDA cores.
 Plan make_plan(int B, int64_t N, int H, int P, int d, sa_dtype dt, bool bwd, bool allow_tc = true) {
   Plan p{};
   const int sms = device_sms() > 0 ? device_sms() : 1;
@@ -136,9 +141,9 @@ sa_status check_args(const void* K, const void* V, const int32_t* cu, int B, int
 
 sa_status check_common(const void* K, const void* V, const int32_t* cu, int B, int64_t N, const void* Q,
                        int H, int P, int d, float scale, sa_dtype dt, const void* ws, size_t ws_bytes,
-                       bool bwd, Plan* plan) {
+                       bool bwd, int uq, Plan* plan) {
   SA_TRY(check_args(K, V, cu, B, N, Q, H, P, d, scale, dt, ws));
-  *plan = make_plan(B, N, H, P, d, dt, bwd, scale >= 0.f);
+  *plan = make_plan(B, N, H, P, d, dt, bwd, scale >= 0.f || !uq);
   if (ws_bytes < plan->lay.total) return SA_ERR_WORKSPACE;
   return SA_OK;
 }
@@ -169,12 +174,32 @@ sa::Args make_args(const void* K, const void* V, const int32_t* cu, int B, int64
   return a;
 }
 
+// A negative scale on the tensor cores: S = scale Q K^T = (-scale) (-Q) K^T,
+// and negating Q is exact, so every score the kernels form -- and the maximum
+// they shift by -- is the one of the caller's problem; the kernels then see a
+// positive scale.  The forward's sketch and lse are unchanged; dK = scale dS Q
+// is unchanged too, while the kernels' dQ is the gradient for -Q, so the caller's
+// dQ is its negation (negate_dq).
+sa_status fold_negative_scale(sa::Args& a, const sa::WsLayout& L, cudaStream_t st) {
+  if (!(a.scale < 0.f)) return SA_OK;
+  void* qn = static_cast<char*>(a.ws) + L.qneg;
+  SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_negate(a.Q, qn, int64_t(a.H) * a.P * a.d, a.dt, st); }));
+  a.Q = qn;
+  a.scale = -a.scale;
+  return SA_OK;
+}
+
+sa_status negate_dq(float* dQ, int H, int P, int d, cudaStream_t st) {
+  return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_negate(dQ, dQ, int64_t(H) * P * d, SA_F32, st); });
+}
+
 }  // namespace
 
 // ------------------------------------------------------- tensor-core helpers
 namespace sa {
 
 bool tc_path_enabled() { return g_path.load() != 1; }
+uint64_t wait_limit_ns() { return g_wait_ns.load(); }
 bool tc_fwd_sliced_selected() { return g_path.load() == 2; }
 
 namespace tcc {
@@ -258,12 +283,13 @@ sa_status fwd_impl(const void* K, const void* V, const int32_t* cu_seqlens, int 
                    size_t ws_bytes, void* stream, int uq) {
   if (!sketch) return SA_ERR_INVALID_ARG;
   Plan plan;
-  SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, false, &plan));
+  SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, false, uq, &plan));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, plan.lay);
   a.uq = uq;
   char* base = static_cast<char*>(workspace);
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, plan.T_fwd, st); }));
+  if (plan.fwd_path == Path::TcFwd) SA_TRY(fold_negative_scale(a, plan.lay, st));
   if (plan.fwd_path == Path::TcFwd) {
     float* l = lse;
     if (sa::tc_fwd_needs_lse_pass_d(P, d)) {
@@ -287,19 +313,22 @@ sa_status bwd_impl(const void* K, const void* V, const int32_t* cu_seqlens, int 
                    void* dV, float* dQ, void* workspace, size_t ws_bytes, void* stream, int uq) {
   if (!dsketch || !dQ || (N > 0 && (!dK || !dV))) return SA_ERR_INVALID_ARG;
   Plan plan;
-  SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, true, &plan));
+  SA_TRY(check_common(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, ws_bytes, true, uq, &plan));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   sa::Args a = make_args(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, workspace, plan.lay);
   a.uq = uq;
   a.dq_user = uq ? dQ : nullptr;
+  const bool folded = plan.bwd_path == Path::TcBwd && scale < 0.f;
   // dQ from the per-worker pieces: summed over workers per head (shared
   // queries) or, per user, only for segments cut across workers
   auto finalize_dq = [&](int W) -> sa_status {
     if (uq) return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_sketch(a, W, dQ, st); });
-    return launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, W, dQ, st); });
+    SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_finalize_dq(a, W, dQ, st); }));
+    return folded ? negate_dq(dQ, H, P, d, st) : SA_OK;
   };
   char* base = static_cast<char*>(workspace);
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, plan.T_bwd, st); }));
+  if (folded) SA_TRY(fold_negative_scale(a, plan.lay, st));
   const float* l = lse;
   if (!l) {
     float* scratch = reinterpret_cast<float*>(base + plan.lay.lse);
@@ -437,7 +466,8 @@ struct TwLayout {
 TwLayout tw_layout(int B, int H, int P, int d, sa_dtype dt, float scale, bool bwd) {
   TwLayout t{};
   const int sms = device_sms() > 0 ? device_sms() : 1;
-  t.tc_fwd = sa::tc_tw_fwd_supported(P, d, dt, scale);
+  // a negative scale is folded into negated prototypes (fold_negative_scale)
+  t.tc_fwd = sa::tc_tw_fwd_supported(P, d, dt, scale < 0.f ? -scale : scale);
   t.tc_bwd = sa::tc_tw_bwd_supported(P, d, dt);
   t.Tf = t.tc_fwd ? sa::tc_tile_tokens() : sa::tw_tile_tokens();
   t.Wf = t.tc_fwd ? sa::tc_tw_fwd_workers(sms, P) : sa::simt_workers(sms, P);
@@ -464,6 +494,8 @@ TwLayout tw_layout(int B, int H, int P, int d, sa_dtype dt, float scale, bool bw
     t.gbf = off;
     if (t.tc_bwd) off = sa::align256(off + 2 * size_t(B) * H * P * d);
   }
+  L.qneg = off;
+  off = sa::align256(off + 4 * size_t(H) * P * d);
   L.lse = L.dcoef = L.gbf = L.lse_part = off;  // unused on this path
   L.total = t.total = off;
   return t;
@@ -478,9 +510,11 @@ sa_status tw_check(const void* K, const void* V, const int32_t* cu, int B, int64
 
 // Plan for the forward's tiles, online-softmax sweep, merge of cut segments:
 // sketch and lse_tok.
-sa_status tw_forward(const sa::Args& a, const TwLayout& lay, float* sketch, float* lse_tok, cudaStream_t st) {
+sa_status tw_forward(const sa::Args& a_in, const TwLayout& lay, float* sketch, float* lse_tok, cudaStream_t st) {
+  sa::Args a = a_in;
   float2* stat = reinterpret_cast<float2*>(static_cast<char*>(a.ws) + lay.stat_part);
   SA_TRY(launch(SA_KERNEL_AUX, st, [&] { return sa::launch_plan(a, lay.Tf, st); }));
+  if (lay.tc_fwd) SA_TRY(fold_negative_scale(a, lay.base, st));  // the backward needs no fold
   if (lay.tc_fwd) {
     SA_TRY(launch(SA_KERNEL_FWD_MAIN, st,
                   [&] { return sa::launch_tc_tw_fwd(a, lay.Wf, sketch, lse_tok, stat, st); }));
@@ -595,6 +629,12 @@ sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches)
 }
 
 uint64_t sa_launch_count(void) { return g_launches.load(); }
+
+sa_status sa_set_wait_limit_ns(uint64_t ns) {
+  if (ns > 60ull * 1000000000ull) return SA_ERR_INVALID_ARG;
+  g_wait_ns.store(ns == 0 ? kDefaultWaitNs : ns);
+  return SA_OK;
+}
 
 sa_status sa_select_path(int path) {
   if (path < 0 || path > 2) return SA_ERR_INVALID_ARG;

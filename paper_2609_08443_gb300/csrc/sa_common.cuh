@@ -31,7 +31,9 @@ struct WsHeader {
   uint32_t pad0;
   int64_t tiles_per_head; // sum_b ceil(L_b / T) for the plan of this call
   uint32_t timeout_site;  // where a bounded wait gave up (diagnostics)
-  uint32_t pad1[59];
+  uint32_t pad1;
+  uint64_t wait_limit_ns; // limit of every bounded pipeline wait of this call
+  uint32_t pad2[56];
 };
 static_assert(sizeof(WsHeader) == 256, "header is one 256-byte line");
 
@@ -46,6 +48,7 @@ struct WsLayout {
   size_t dcoef;        // fp32 [N][H]: D_i = dV_i . v_i (bwd)
   size_t gbf;          // bf16 [B][H][P][d]: dsketch copy streamed by TMA (bwd, d = 128)
   size_t lse_part;     // float2 [N][H][P / 512]: per-slice (max, sum) of the lse pass (P >= 1024)
+  size_t qneg;         // [H][P][d] (4 bytes per element reserved): -Q, for a negative scale
   size_t total;
 };
 
@@ -66,6 +69,8 @@ SA_HD WsLayout ws_layout(int B, int64_t N, int H, int P, int d, int W, bool bwd)
   if (bwd && d == 128 && P > 128) off = align256(off + 2 * size_t(B) * size_t(H) * size_t(P) * size_t(d));
   L.lse_part = off;
   if (P >= 1024) off = align256(off + 8 * size_t(N) * size_t(H) * size_t((P + 511) / 512));
+  L.qneg = off;
+  off = align256(off + 4 * size_t(H) * size_t(P) * size_t(d));
   L.total = off;
   return L;
 }

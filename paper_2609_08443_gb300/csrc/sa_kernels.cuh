@@ -28,6 +28,10 @@ struct Args {
 // Row of Q ([H or B*H][P][d]) that user b, head h reads.
 SA_HD int q_row(const Args& a, int b, int h) { return a.uq ? b * a.H + h : h; }
 
+// Limit of the bounded pipeline waits for calls enqueued from now on
+// (sa_set_wait_limit_ns; the planner copies it into each call's workspace).
+uint64_t wait_limit_ns();
+
 // planner / finalize (sa_simt.cu)
 cudaError_t launch_plan(const Args& a, int T, cudaStream_t st);
 cudaError_t launch_finalize_sketch(const Args& a, int W, float* sketch, cudaStream_t st);
@@ -37,6 +41,8 @@ cudaError_t launch_finalize_dq(const Args& a, int W, float* dQ, cudaStream_t st)
 cudaError_t launch_fold_wk(const void* Q, const void* Wk, int H, int P, int d, sa_dtype dt, void* Qf,
                            cudaStream_t st);
 cudaError_t launch_add_into(void* dX, const void* dKf, int64_t n, sa_dtype dt, cudaStream_t st);
+// dst = -src, n elements of type dt (src == dst allowed)
+cudaError_t launch_negate(const void* src, void* dst, int64_t n, sa_dtype dt, cudaStream_t st);
 cudaError_t launch_wk_grads(const float* dQf, const void* Q, const void* Wk, int H, int P, int d, sa_dtype dt,
                             float* dQ, float* dWk, cudaStream_t st);
 

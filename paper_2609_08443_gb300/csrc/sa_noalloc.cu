@@ -8,6 +8,8 @@
 // scratch from a fixed array that lives in this library's device image.
 #include <mutex>
 
+#include <cuda.h>
+
 #include "sa_kernels.cuh"
 
 namespace {
@@ -18,22 +20,51 @@ constexpr size_t kNoAllocScratchBytes = size_t(32) << 20;  // 32 MiB
 
 __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-std::mutex g_noalloc_mu;
-void* g_noalloc_addr[64] = {nullptr};
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
 
-// Device address of the array on the current device.  In host code the
-// array's name is only a host-side stand-in, so the real address is looked up
-// once per device (with that device current) and cached.
+CtxGetCurrentFn ctx_get_current_fn() {
+  static CtxGetCurrentFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  });
+  return fn;
+}
+
+struct ScratchAddr {
+  CUcontext ctx = nullptr;
+  void* ptr = nullptr;
+};
+std::mutex g_noalloc_mu;
+ScratchAddr g_noalloc_addr[64];
+
+// Device address of the array in the current device's context.  In host code
+// the array's name is only a host-side stand-in, so the real address is looked
+// up with the device current and cached per device, together with the context
+// it belongs to: after a device reset the context changes and the address is
+// looked up again instead of reusing one that points into freed memory.
 sa_status noalloc_scratch(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SA_ERR_CUDA;
+  CtxGetCurrentFn get = ctx_get_current_fn();
+  if (!get) return SA_ERR_CUDA;
+  CUcontext ctx = nullptr;  // null until the runtime has made a context current in this thread
+  if (get(&ctx) != CUDA_SUCCESS) return SA_ERR_CUDA;
   std::lock_guard<std::mutex> lk(g_noalloc_mu);
-  if (g_noalloc_addr[dev] == nullptr) {
+  ScratchAddr& c = g_noalloc_addr[dev];
+  if (ctx == nullptr || c.ptr == nullptr || c.ctx != ctx) {
+    // the lookup makes the device's primary context current if none is
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return SA_ERR_CUDA;
-    g_noalloc_addr[dev] = p;
+    if (get(&ctx) != CUDA_SUCCESS || ctx == nullptr) return SA_ERR_CUDA;
+    c.ctx = ctx;
+    c.ptr = p;
   }
-  *out = g_noalloc_addr[dev];
+  *out = c.ptr;
   return SA_OK;
 }
 
@@ -52,11 +83,19 @@ sa_status sa_sketch_fwd_noalloc(const void* K, const void* V, const int32_t* cu_
   void* scratch = nullptr;
   const sa_status st = noalloc_scratch(&scratch);
   if (st != SA_OK) return st;
-  // The planner kernel rewrites the array's header (error word, tile counts)
-  // at the start of every call, and every other section is written before it
-  // is read within the call, so nothing carried over from the last call is used.
+  // The planner kernel rewrites the array's header (error word, tile counts,
+  // wait limit) at the start of every call, and every other section is written
+  // before it is read within the call, so nothing carried over from the last
+  // call is used -- including the error word of a call that failed.
   return sa_sketch_fwd(K, V, cu_seqlens, B, N, Q, H, P, d, scale, dt, sketch, lse, scratch,
                        kNoAllocScratchBytes, stream);
+}
+
+sa_status sa_noalloc_get_device_error(void* stream) {
+  void* scratch = nullptr;
+  const sa_status st = noalloc_scratch(&scratch);
+  if (st != SA_OK) return st;
+  return sa_get_device_error(scratch, stream);
 }
 
 }  // extern "C"

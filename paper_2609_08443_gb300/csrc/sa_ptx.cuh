@@ -45,21 +45,26 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Every wait in the tensor-core kernels is bounded: after kWaitLimitNs the
+// Every wait in the tensor-core kernels is bounded: after the call's limit
+// (the workspace header's wait_limit_ns, 2 s unless a test lowers it) the
 // waiting thread raises the CTA's abort flag and records SA_ERR_TIMEOUT in the
 // workspace; threads that see the flag stop waiting too.  A correct pipeline
 // never gets near the limit.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 
+__device__ __forceinline__ uint64_t wait_limit(const void* ws) {
+  return reinterpret_cast<const volatile WsHeader*>(ws)->wait_limit_ns;
+}
+
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, void* ws,
                                           uint32_t site) {
   if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
+  const uint64_t t0 = globaltimer(), lim = wait_limit(ws);
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63u) == 0u) {
       if (*abort_flag) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
+      if (globaltimer() - t0 > lim) {
         *abort_flag = 1;
         ws_set_error(ws, SA_ERR_TIMEOUT, site);
         return false;
@@ -131,12 +136,12 @@ __device__ __forceinline__ void cluster_sync_all() {
 __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, volatile int* abort_flag, void* ws,
                                                   uint32_t site) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
+  const uint64_t t0 = globaltimer(), lim = wait_limit(ws);
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
     if ((it & 63u) == 0u) {
       if (*abort_flag) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
+      if (globaltimer() - t0 > lim) {
         *abort_flag = 1;
         ws_set_error(ws, SA_ERR_TIMEOUT, site);
         return false;

@@ -20,7 +20,7 @@ constexpr int SNT = 256;  // threads per block
 // One block: validates cu_seqlens and writes the per-head tile prefix.
 __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ cu, int B,
                                                     int64_t N, int T, void* ws,
-                                                    int64_t* __restrict__ prefix) {
+                                                    int64_t* __restrict__ prefix, uint64_t wait_ns) {
   __shared__ int64_t warp_tot[32];
   __shared__ int64_t carry;
   __shared__ int bad;
@@ -29,6 +29,7 @@ __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ 
     carry = 0;
     bad = (cu[0] != 0) || (int64_t(cu[B]) != N);
     ws_header(ws)->timeout_site = 0;
+    ws_header(ws)->wait_limit_ns = wait_ns;
   }
   __syncthreads();
   for (int base = 0; base < B; base += 1024) {
@@ -497,7 +498,7 @@ static size_t smem_bwd_tok(int d) { return sizeof(float) * (size_t(2 * ST + 2 * 
 static size_t smem_bwd_dq(int d) { return smem_bwd_tok(d); }
 
 cudaError_t launch_plan(const Args& a, int T, cudaStream_t st) {
-  plan_kernel<<<1, 1024, 0, st>>>(a.cu, a.B, a.N, T, a.ws, a.prefix);
+  plan_kernel<<<1, 1024, 0, st>>>(a.cu, a.B, a.N, T, a.ws, a.prefix, wait_limit_ns());
   return cudaGetLastError();
 }
 

@@ -185,9 +185,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         it.next();
       }
-      if (!ok) {
+      if (!ok) {  // drain the ring loads and the prototype block still in flight
         for (uint32_t k = (e > uint32_t(C::NSLOT) ? e - C::NSLOT : 0); k < e; ++k)
           mbar_wait_bounded(ring_full(int(k % C::NSLOT)), (k / C::NSLOT) & 1, 200000000ull);
+        if (hc > 0) mbar_wait_bounded(q_full, uint32_t(hc - 1) & 1u, 200000000ull);
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- UMMA issuer

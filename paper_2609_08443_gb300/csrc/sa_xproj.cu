@@ -45,6 +45,13 @@ __global__ void add_into_kernel(T* __restrict__ dX, const T* __restrict__ dKf, i
     st_from_f32(dX + i, ld_f32(dX + i) + ld_f32(dKf + i));
 }
 
+// dst = -src elementwise (exact in bf16 and fp32).
+template <typename T>
+__global__ void negate_kernel(const T* __restrict__ src, T* __restrict__ dst, int64_t n) {
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n; i += int64_t(gridDim.x) * blockDim.x)
+    dst[i] = -src[i];
+}
+
 // dQ[h] = dQ'[h] Wk[h]  (P x d),  dWk[h] = dQ'[h]^T Q[h]  (d x d); fp32 outputs.
 // grid (ceil(max(P, d) / 8), H); each block computes 8 rows of both.
 template <typename T>
@@ -90,6 +97,17 @@ cudaError_t launch_add_into(void* dX, const void* dKf, int64_t n, sa_dtype dt, c
                                                          static_cast<const __nv_bfloat16*>(dKf), n);
   else
     add_into_kernel<float><<<2048, 256, 0, st>>>(static_cast<float*>(dX), static_cast<const float*>(dKf), n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_negate(const void* src, void* dst, int64_t n, sa_dtype dt, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  const int blocks = int((n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024);
+  if (dt == SA_BF16)
+    negate_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(src),
+                                                         static_cast<__nv_bfloat16*>(dst), n);
+  else
+    negate_kernel<float><<<blocks, 256, 0, st>>>(static_cast<const float*>(src), static_cast<float*>(dst), n);
   return cudaGetLastError();
 }
 

@@ -107,6 +107,18 @@ def step_work(tokens, B, H, P, d, elem_bytes) -> Work:
                 recompute_flops=b.recompute_flops)
 
 
+# MUFU exp2 throughput of one GB300 SM, in ex2.approx results per SM clock.
+# Measured on the GB300s: a grid of 8 blocks of 256 threads per SM,
+# each thread running 8 independent chains x <- 2^-x, timed with CUDA events
+# over 2000 back-to-back launches; rate / (SMs x maximum SM clock).
+EX2_PER_SM_CLK = 31.0
+
+
+def exp_peak_per_s(num_sms: int, sm_mhz: float) -> float:
+    """MUFU exp2 peak of the whole GPU at the given SM clock."""
+    return EX2_PER_SM_CLK * num_sms * sm_mhz * 1e6
+
+
 def roofline_time(work: Work, peak_tflops: float, peak_gbs: float,
                   exp_per_s: Optional[float] = None) -> Dict[str, float]:
     """Slowest of the tensor, HBM and exp bounds, in seconds."""

@@ -74,3 +74,15 @@ def check_spec(spec, bwd=True, pass_lse=True, users=None, per_user_q=False):
     if host["K"].shape[0]:
         assert np.max(np.abs(got["lse"] - ref["lse"])) <= 5e-3 * max(1.0, np.max(np.abs(ref["lse"])))
     return errs
+
+
+def oracle_dq_chunk(job):
+    """dQ [H, P, d] of one piece of one user's history (bf16 bit patterns of K
+    and V, fp64 Q and that user's dsketch [H, P, d]).  The prototype-wise weights
+    are per token, so a user's dQ is the sum of its pieces' dQ; worker function
+    of the full-batch tests' process pool."""
+    kbits, vbits, Q, G, scale = job
+    K = wl.bf16_bits_to_f64(kbits)
+    V = wl.bf16_bits_to_f64(vbits)
+    _, _, dQ = sa_backward(K, V, np.array([0, K.shape[0]]), Q, scale, G[None])
+    return dQ

@@ -152,3 +152,9 @@ def test_step_host_checks(lib):
                                  vp(3072), vp(4096), vp(8192), vp(9216), 0, vp(1 << 20), 16, None)
     assert st == 3
     assert lib.sa_step_host_workspace_size(cu.ctypes.data, 2, 1, 64, 64, 1, 0) > 0
+
+
+def test_wait_limit_bounds(lib):
+    assert lib.sa_set_wait_limit_ns(61 * 10**9) == 1  # above 60 s: SA_ERR_INVALID_ARG
+    assert lib.sa_set_wait_limit_ns(5 * 10**9) == 0
+    assert lib.sa_set_wait_limit_ns(0) == 0           # back to the default

@@ -89,7 +89,8 @@ def test_large_p_100k_user(cuda_lib):
 @pytest.mark.parametrize("P,d", [(512, 128), (256, 64)])
 def test_negative_scale(cuda_lib, P, d):
     """A negative scale (valid; the softmax then favours anti-aligned keys) runs on
-    the CUDA-core kernels: same parity bar."""
+    the tensor-core kernels, its sign folded into a negated copy of Q: same
+    parity bar."""
     spec = wl.custom(RAGGED, H=2, P=P, d=d, dtype=wl.BF16, seed=P + d + 5)
     host = wl.make_host(spec)
     t = wl.host_to_torch(spec, host, torch.device("cuda"))

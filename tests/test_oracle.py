@@ -49,3 +49,21 @@ def test_oracle_tokenwise_pin(pin):
     if pin.__name__.endswith("bruteforce"):
         pytest.importorskip("mpmath")
     pin(sa_forward_tokenwise, sa_backward_tokenwise)
+
+
+def test_dq_is_a_sum_over_pieces_of_a_history():
+    """Prototype-wise weights are per token, so a user's dQ is the sum of the dQ
+    of any split of its tokens into pieces (the full-batch GPU tests sum the
+    oracle's dQ this way)."""
+    import harness
+    from paper_2609_08443_gb300 import workloads as wl
+
+    spec = wl.custom([37], H=2, P=5, d=8, dtype=wl.BF16, seed=9)
+    host = wl.make_host(spec)
+    Q = wl.host_as_f64(spec, host["Q"])
+    G = host["dsketch"].astype(np.float64)
+    K, V = wl.host_as_f64(spec, host["K"]), wl.host_as_f64(spec, host["V"])
+    _, _, dq_all = sa_backward(K, V, host["cu_seqlens"], Q, spec.scale, G)
+    parts = sum(harness.oracle_dq_chunk((host["K"][s:e], host["V"][s:e], Q, G[0], spec.scale))
+                for s, e in ((0, 10), (10, 11), (11, 37)))
+    assert np.max(np.abs(parts - dq_all)) <= 1e-12 * np.max(np.abs(dq_all))
