@@ -214,7 +214,12 @@ sa_status sa_sketch_step_host(const void* K, const void* V, const int32_t* cu_se
  * of sa_noalloc_scratch_bytes() bytes (32 MiB) that this library keeps in
  * device memory on every GPU where it is loaded, until the process exits.
  *   - Returns SA_ERR_WORKSPACE, before launching anything, when the call would
- *     need more scratch than that (large N, B, P or d); use sa_sketch_fwd then.
+ *     need more scratch than that; use sa_sketch_fwd then.  The scratch holds
+ *     per-worker sketch pieces (2 x P x d fp32 per SM) and per-token
+ *     statistics (4 bytes per token and head), so on a 152-SM GB300 the array
+ *     serves, for example, P = 256 with d = 64 or P = 128 with d = 128 for
+ *     batches of up to about 3 million token-heads (tokens x heads); the
+ *     100K-token workload's P = 512 with d = 128 does not fit.
  *   - It allocates nothing itself.  The array belongs to the current device
  *     (cudaGetDevice), not to the device of `stream` or of the tensors: make
  *     the device that owns the stream and all buffers current before calling.
@@ -281,7 +286,7 @@ uint64_t sa_launch_count(void);
 
 /* Time limit, in nanoseconds, of every bounded wait inside the tensor-core
  * kernels, for calls enqueued after this one (0 restores the default of 2 s;
- * at most 60 s, else SA_ERR_INVALID_ARG).  A correct pipeline never waits
+ * at most 4 s, else SA_ERR_INVALID_ARG).  A correct pipeline never waits
  * anywhere near 2 s; a lower limit exists so that tests can make a wait run
  * out on purpose and check the recovery: the call's kernels stop, drain their
  * copies and tensor-core work still in flight, release their tensor memory,

@@ -631,7 +631,7 @@ sa_status sa_timing_read(sa_kernel_class k, double* total_ms, int64_t* launches)
 uint64_t sa_launch_count(void) { return g_launches.load(); }
 
 sa_status sa_set_wait_limit_ns(uint64_t ns) {
-  if (ns > 60ull * 1000000000ull) return SA_ERR_INVALID_ARG;
+  if (ns > 4000000000ull) return SA_ERR_INVALID_ARG;
   g_wait_ns.store(ns == 0 ? kDefaultWaitNs : ns);
   return SA_OK;
 }

@@ -46,7 +46,7 @@ struct WsLayout {
   size_t dq_partial;   // fp32 [W][H][P][d]: per-worker dQ per head (bwd)
   size_t lse;          // fp32 [N][H]: lse scratch when the caller passes none
   size_t dcoef;        // fp32 [N][H]: D_i = dV_i . v_i (bwd)
-  size_t gbf;          // bf16 [B][H][P][d]: dsketch copy streamed by TMA (bwd, d = 128)
+  size_t gbf;          // bf16 [B][H][P][d]: dsketch copy streamed by TMA (split backward)
   size_t lse_part;     // float2 [N][H][P / 512]: per-slice (max, sum) of the lse pass (P >= 1024)
   size_t qneg;         // [H][P][d] (4 bytes per element reserved): -Q, for a negative scale
   size_t total;
@@ -66,7 +66,8 @@ SA_HD WsLayout ws_layout(int B, int64_t N, int H, int P, int d, int W, bool bwd)
   L.dcoef = off;
   if (bwd) off = align256(off + sizeof(float) * size_t(N) * size_t(H));
   L.gbf = off;
-  if (bwd && d == 128 && P > 128) off = align256(off + 2 * size_t(B) * size_t(H) * size_t(P) * size_t(d));
+  if (bwd && ((d == 128 && P > 128) || (d == 64 && P > 256)))
+    off = align256(off + 2 * size_t(B) * size_t(H) * size_t(P) * size_t(d));
   L.lse_part = off;
   if (P >= 1024) off = align256(off + 8 * size_t(N) * size_t(H) * size_t((P + 511) / 512));
   L.qneg = off;

@@ -50,26 +50,56 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 // waiting thread raises the CTA's abort flag and records SA_ERR_TIMEOUT in the
 // workspace; threads that see the flag stop waiting too.  A correct pipeline
 // never gets near the limit.
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
+//
+// Each CTA keeps two control words in shared memory, reached through the
+// `abort_flag` pointer every wait takes: abort_flag[0] is the abort flag and
+// abort_flag[2] the limit in nanoseconds, copied from the workspace header by
+// wait_ctl_init when the CTA starts (abort_flag[1] is left to the kernel).
 
-__device__ __forceinline__ uint64_t wait_limit(const void* ws) {
-  return reinterpret_cast<const volatile WsHeader*>(ws)->wait_limit_ns;
+__device__ __forceinline__ void wait_ctl_init(volatile int* abort_flag, const void* ws) {
+  const uint64_t ns = reinterpret_cast<const WsHeader*>(ws)->wait_limit_ns;
+  abort_flag[0] = 0;
+  reinterpret_cast<volatile uint32_t*>(abort_flag)[2] = ns > 0xFFFFFFFFull ? 0xFFFFFFFFu : uint32_t(ns);
+}
+
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Limits below this are test settings: the wait then polls without suspending
+// so that it gives up within a few hundred nanoseconds of the limit.
+constexpr uint32_t kPollLimitNs = 1000000u;  // 1 ms
+
+__device__ __forceinline__ bool mbar_wait_timed_out(volatile int* abort_flag, void* ws, uint32_t site, uint64_t t0,
+                                                    uint64_t lim) {
+  if (globaltimer() - t0 <= lim) return false;
+  *abort_flag = 1;
+  ws_set_error(ws, SA_ERR_TIMEOUT, site);
+  return true;
 }
 
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, void* ws,
                                           uint32_t site) {
   if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer(), lim = wait_limit(ws);
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 0u) {
-      if (*abort_flag) return false;
-      if (globaltimer() - t0 > lim) {
-        *abort_flag = 1;
-        ws_set_error(ws, SA_ERR_TIMEOUT, site);
-        return false;
-      }
+  const uint64_t t0 = globaltimer();
+  const uint32_t lim = reinterpret_cast<volatile const uint32_t*>(abort_flag)[2];
+  if (lim < kPollLimitNs) {
+    for (;;) {
+      if (mbar_test_wait(bar, parity)) return true;
+      if (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim)) return false;
     }
+  }
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim)) return false;
   }
 }
 
@@ -136,17 +166,11 @@ __device__ __forceinline__ void cluster_sync_all() {
 __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, volatile int* abort_flag, void* ws,
                                                   uint32_t site) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
-  const uint64_t t0 = globaltimer(), lim = wait_limit(ws);
-  for (uint32_t it = 1;; ++it) {
+  const uint64_t t0 = globaltimer();
+  const uint32_t lim = reinterpret_cast<volatile const uint32_t*>(abort_flag)[2];
+  for (;;) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
-    if ((it & 63u) == 0u) {
-      if (*abort_flag) return false;
-      if (globaltimer() - t0 > lim) {
-        *abort_flag = 1;
-        ws_set_error(ws, SA_ERR_TIMEOUT, site);
-        return false;
-      }
-    }
+    if (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim)) return false;
   }
 }
 

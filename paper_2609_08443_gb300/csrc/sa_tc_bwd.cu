@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(dq_full, 1);
     mbar_init(dq_empty, kSoftWarps);
     mbar_init(drain, 1);
-    *abort_flag = 0;
+    wait_ctl_init(abort_flag, a.ws);
     fence_mbar_init();
   }
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
@@ -563,14 +563,17 @@ static cudaError_t launch_bwd_t(const Args& a, int W, const float* dsk, const fl
 }  // namespace tcb
 
 // Tensor-core backward: bf16, all prototypes in one CTA when the four TMEM
-// accumulators fit (d = 64 with P <= 256, d = 128 with P = 128).
+// accumulators fit (d = 64 with P <= 256, d = 128 with P = 128), else the
+// token-side kernel plus the dQ slices (tc_bwd_split).
 bool tc_bwd_supported(int P, int d, sa_dtype dt) {
   if (dt != SA_BF16 || !tcc::device_is_sm103() || !tc_path_enabled()) return false;
-  return (d == 64 && (P == 128 || P == 256)) ||
-         (d == 128 && (P == 128 || P == 256 || P == 512 || P == 1024 || P == 2048));
+  return ((d == 64 || d == 128) && (P == 128 || P == 256 || P == 512 || P == 1024 || P == 2048));
 }
 
 const char* tc_bwd_name(int P, int d) {
+  if (d == 64 && P == 2048) return "tc_bwd_tok_kernel<64,2048>";
+  if (d == 64 && P == 1024) return "tc_bwd_tok_kernel<64,1024>";
+  if (d == 64 && P == 512) return "tc_bwd_tok_kernel<64,512>";
   if (d == 64) return P == 256 ? "tc_bwd_kernel<64,256,full>" : "tc_bwd_kernel<64,128,full>";
   if (P == 2048) return "tc_bwd_tok_kernel<128,2048>";
   if (P == 1024) return "tc_bwd_tok_kernel<128,1024>";
@@ -702,7 +705,7 @@ __device__ __forceinline__ void bwd_tok_body(const CUtensorMap& tmK, const CUten
     mbar_init(epi_ready, kSoftWarps);
     mbar_init(epi_free, 1);
     mbar_init(drain, 1);
-    *abort_flag = 0;
+    wait_ctl_init(abort_flag, a.ws);
     fence_mbar_init();
   }
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
@@ -1162,7 +1165,10 @@ static cudaError_t launch_tok_t(const Args& a, int W, const __nv_bfloat16* gbf, 
 
 }  // namespace tcb
 
-bool tc_bwd_split(int P, int d) { return d == 128 && (P == 256 || P == 512 || P == 1024 || P == 2048); }
+bool tc_bwd_split(int P, int d) {
+  return (d == 128 && (P == 256 || P == 512 || P == 1024 || P == 2048)) ||
+         (d == 64 && (P == 512 || P == 1024 || P == 2048));
+}
 
 cudaError_t launch_tc_g_bf16(const Args& a, const float* dsk, __nv_bfloat16* gbf, cudaStream_t st) {
   const int64_t n8 = int64_t(a.B) * a.H * a.P * a.d / 8;
@@ -1174,6 +1180,11 @@ cudaError_t launch_tc_bwd_tok(const Args& a, int W, const float* dsk, __nv_bfloa
                               float* Dco, void* dK, void* dV, cudaStream_t st) {
   (void)dsk;
   if (a.N == 0) return cudaSuccess;
+  if (a.d == 64) {
+    if (a.P == 2048) return tcb::launch_tok_t<64, 2048>(a, W, gbf, lse, Dco, dK, dV, st);
+    if (a.P == 1024) return tcb::launch_tok_t<64, 1024>(a, W, gbf, lse, Dco, dK, dV, st);
+    return tcb::launch_tok_t<64, 512>(a, W, gbf, lse, Dco, dK, dV, st);
+  }
   if (a.P == 2048) return tcb::launch_tok_t<128, 2048>(a, W, gbf, lse, Dco, dK, dV, st);
   if (a.P == 1024) return tcb::launch_tok_t<128, 1024>(a, W, gbf, lse, Dco, dK, dV, st);
   if (a.P == 512) return tcb::launch_tok_t<128, 512>(a, W, gbf, lse, Dco, dK, dV, st);
@@ -1290,7 +1301,7 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
     mbar_init(col_empty0, kSoftWarps);
     mbar_init(col_empty0 + 8, kSoftWarps);
     mbar_init(drain, 1);
-    *abort_flag = 0;
+    wait_ctl_init(abort_flag, a.ws);
     fence_mbar_init();
   }
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
@@ -1648,7 +1659,7 @@ namespace sa {
 cudaError_t launch_tc_bwd_dq(const Args& a, int W, const float* dsk, const float* lse, const float* Dco,
                              cudaStream_t st) {
   if (a.N == 0) return cudaSuccess;
-  return tcb::launch_dq_t<128, 128>(a, W, dsk, lse, Dco, st);
+  return a.d == 64 ? tcb::launch_dq_t<64, 128>(a, W, dsk, lse, Dco, st) : tcb::launch_dq_t<128, 128>(a, W, dsk, lse, Dco, st);
 }
 
 // Token-wise normalisation (Sec. 5.1): the same two kernels with per-prototype

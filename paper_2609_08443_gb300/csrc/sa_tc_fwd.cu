@@ -138,7 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(st_used, kSoftWarps);
     mbar_init(r_full, 1);
     mbar_init(r_used, kSoftWarps);
-    *abort_flag = 0;
+    wait_ctl_init(abort_flag, a.ws);
     *skip_flag = skip ? 1u : 0u;
     fence_mbar_init();
   }
@@ -545,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(drain, 1);
     mbar_init(st_ready, kSoftWarps);
     mbar_init(st_used, kSoftWarps);
-    *abort_flag = 0;
+    wait_ctl_init(abort_flag, a.ws);
     fence_mbar_init();
   }
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);

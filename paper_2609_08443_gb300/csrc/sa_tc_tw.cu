@@ -105,7 +105,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(o_full, 1);
     mbar_init(o_empty, C::SOFT_WARPS);
     mbar_init(drain, 1);
-    *abort_flag = 0;
+    wait_ctl_init(abort_flag, a.ws);
     fence_mbar_init();
   }
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);

@@ -246,7 +246,7 @@ def make_device(spec: Spec, device="cuda"):
     K = normal((N, spec.H, spec.d))
     V = normal((N, spec.H, spec.d))
     Q = normal((spec.H, spec.P, spec.d), spec.q_std)
-    dS = torch.randn((spec.B, spec.H, spec.P, spec.d), generator=g, device=device,
+    dS = torch.randn((lens.size, spec.H, spec.P, spec.d), generator=g, device=device,
                      dtype=torch.float32)
     return {"K": K, "V": V, "Q": Q, "cu_seqlens": torch.from_numpy(cu).to(device),
             "dsketch": dS, "lengths": lens}
