@@ -201,6 +201,7 @@ namespace sa {
 bool tc_path_enabled() { return g_path.load() != 1; }
 uint64_t wait_limit_ns() { return g_wait_ns.load(); }
 bool tc_fwd_sliced_selected() { return g_path.load() == 2; }
+bool tc_fwd_pair_selected() { return g_path.load() == 3; }
 
 namespace tcc {
 
@@ -637,7 +638,7 @@ sa_status sa_set_wait_limit_ns(uint64_t ns) {
 }
 
 sa_status sa_select_path(int path) {
-  if (path < 0 || path > 2) return SA_ERR_INVALID_ARG;
+  if (path < 0 || path > 3) return SA_ERR_INVALID_ARG;
   g_path.store(path);
   return SA_OK;
 }

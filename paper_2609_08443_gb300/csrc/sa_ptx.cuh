@@ -97,9 +97,11 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
       if (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim)) return false;
     }
   }
-  for (;;) {
+  // the flag and the clock are checked every 64 polls: a handoff that is not
+  // ready at the first poll is then noticed as soon as it completes
+  for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim)) return false;
+    if ((it & 63u) == 0u && (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim))) return false;
   }
 }
 
@@ -168,9 +170,9 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity,
   if (mbar_try_wait_cluster(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   const uint32_t lim = reinterpret_cast<volatile const uint32_t*>(abort_flag)[2];
-  for (;;) {
+  for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
-    if (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim)) return false;
+    if ((it & 63u) == 0u && (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim))) return false;
   }
 }
 

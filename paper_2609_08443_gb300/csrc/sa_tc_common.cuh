@@ -131,8 +131,9 @@ __device__ __forceinline__ void store_sketch(uint32_t tmem, uint32_t lane_off, i
       const int pbase = sw * (PS / 2) + 32 * c;
       ptx::tmem_ld32(tmem + lane_off + O_COL + pbase, v);
       ptx::tmem_ld_wait();
+      float* col = dst + int64_t(pbase) * D + d;  // prototype pbase, feature d; the next prototype is D floats on
 #pragma unroll
-      for (int k = 0; k < 32; ++k) dst[int64_t(pbase + k) * D + d] = v[k];
+      for (int k = 0; k < 32; ++k) col[k * D] = v[k];
     }
   } else {
     constexpr int NB = PS / 128;

@@ -16,8 +16,7 @@ def test_tensor_core_path_matches_cuda_core_path(cuda_lib, P, d):
     host = wl.make_host(spec)
     t = wl.host_to_torch(spec, host, torch.device("cuda"))
     assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, False).startswith("tc_")
-    if (d == 64 and P <= 256) or d == 128:  # d = 64 with P >= 512: CUDA-core backward
-        assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, True).startswith("tc_")
+    assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, True).startswith("tc_")
     tc = harness.gpu_outputs(spec, t, bwd=True)
     binding.sa_select_path(1)
     try:
@@ -51,3 +50,28 @@ def test_pair_forward_matches_lse_pass_and_slices(cuda_lib, P, d):
     assert "sliced" not in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
     assert harness.rel_err(fused["sketch"], sliced["sketch"]) <= 2e-2
     assert abs(fused["lse"] - sliced["lse"]).max() <= 5e-3 * max(1.0, abs(sliced["lse"]).max())
+
+
+@pytest.mark.parametrize("P,d", [(512, 128), (512, 64)])
+def test_pipelined_pair_forward_matches_unpipelined(cuda_lib, P, d):
+    """The software-pipelined cluster-pair forward (tile i's (max, sum) exchange
+    overlapped with tile i+1's scores) against the same pair split without the
+    pipeline, on ragged users that end tiles, segments and worker ranges at
+    every offset; the pipelined kernel is also bitwise reproducible."""
+    spec = wl.custom([700, 0, 128, 129, 3000, 1, 5000, 2, 255, 257], H=3, P=P, d=d, dtype=wl.BF16, seed=P + d + 1)
+    host = wl.make_host(spec)
+    t = wl.host_to_torch(spec, host, torch.device("cuda"))
+    assert "pipe" in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
+    pipe = harness.gpu_outputs(spec, t, bwd=False)
+    pipe2 = harness.gpu_outputs(spec, t, bwd=False)
+    binding.sa_select_path(3)
+    try:
+        assert "pair" in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
+        pair = harness.gpu_outputs(spec, t, bwd=False)
+    finally:
+        binding.sa_select_path(0)
+    assert (pipe["sketch"] == pipe2["sketch"]).all() and (pipe["lse"] == pipe2["lse"]).all()
+    assert harness.rel_err(pipe["sketch"], pair["sketch"]) <= 2e-2
+    assert abs(pipe["lse"] - pair["lse"]).max() <= 5e-3 * max(1.0, abs(pair["lse"]).max())
+    ref = harness.oracle_outputs(spec, host, bwd=False)
+    harness.assert_close("sketch", pipe["sketch"], ref["sketch"], harness.TOL[wl.BF16])
