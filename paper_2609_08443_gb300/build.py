@@ -19,7 +19,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT, "libsa_sketch.so")
-SOURCES = ["sa_api.cu", "sa_simt.cu", "sa_tc_fwd.cu", "sa_tc_fwd_pipe.cu", "sa_tc_bwd.cu", "sa_noalloc.cu", "sa_xproj.cu", "sa_tokenwise.cu", "sa_tc_tw.cu", "sa_host_step.cu"]
+SOURCES = ["sa_api.cu", "sa_simt.cu", "sa_tc_fwd.cu", "sa_tc_fwd_wide.cu", "sa_tc_bwd.cu", "sa_noalloc.cu", "sa_xproj.cu", "sa_tokenwise.cu", "sa_tc_tw.cu", "sa_host_step.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr",
          "-Xptxas", "-warn-spills"]

@@ -9,9 +9,9 @@ bool tc_fwd_needs_lse_pass_d(int P, int d);  // lse pass, then 256-prototype sli
 int tc_lse_slice(int P, int d);              // prototypes per slice of the lse pass
 bool tc_path_enabled();
 bool tc_fwd_sliced_selected();  // sa_select_path(2)
-bool tc_fwd_pair_selected();    // sa_select_path(3): the un-pipelined pair kernel for P = 512
-// P = 512: the software-pipelined cluster-pair forward (sa_tc_fwd_pipe.cu)
-cudaError_t launch_tc_fwd_pipe(const Args& a, int W, float* sketch, float* lse, cudaStream_t st);
+bool tc_fwd_pair_selected();    // sa_select_path(3): the 8-softmax-warp pair kernel for P = 512
+// P = 512: the cluster-pair forward with 16 softmax warps (sa_tc_fwd_wide.cu)
+cudaError_t launch_tc_fwd_wide(const Args& a, int W, float* sketch, float* lse, cudaStream_t st);
 bool tc_bwd_supported(int P, int d, sa_dtype dt);
 const char* tc_fwd_name(int P, int d);
 const char* tc_bwd_name(int P, int d);

@@ -787,7 +787,7 @@ bool tc_fwd_needs_lse_pass_d(int P, int d) {
 
 const char* tc_fwd_name(int P, int d) {
   if (tc_fwd_needs_lse_pass_d(P, d)) return d == 128 ? "tc_fwd_kernel<128,256,sliced>" : "tc_fwd_kernel<64,256,sliced>";
-  if (P == 512 && !tc_fwd_pair_selected()) return d == 128 ? "tc_fwd_pipe_kernel<128>" : "tc_fwd_pipe_kernel<64>";
+  if (P == 512 && !tc_fwd_pair_selected()) return d == 128 ? "tc_fwd_wide_kernel<128>" : "tc_fwd_wide_kernel<64>";
   if (P == 512) return d == 128 ? "tc_fwd_kernel<128,256,pair>" : "tc_fwd_kernel<64,256,pair>";
   if (P == 256) return d == 128 ? "tc_fwd_kernel<128,256,fused>" : "tc_fwd_kernel<64,256,fused>";
   return d == 128 ? "tc_fwd_kernel<128,128,fused>" : "tc_fwd_kernel<64,128,fused>";
@@ -830,7 +830,7 @@ cudaError_t launch_tc_fwd(const Args& a, int W, float* sketch, float* lse, cudaS
   if (tc_fwd_needs_lse_pass_d(a.P, a.d))  // lse (from launch_tc_lse beforehand) is an input here
     return a.d == 128 ? launch_fwd_t<128, 256, kSliced>(a, W, sketch, nullptr, lse, st)
                       : launch_fwd_t<64, 256, kSliced>(a, W, sketch, nullptr, lse, st);
-  if (a.P == 512 && !tc_fwd_pair_selected()) return launch_tc_fwd_pipe(a, W, sketch, lse, st);
+  if (a.P == 512 && !tc_fwd_pair_selected()) return launch_tc_fwd_wide(a, W, sketch, lse, st);
   if (a.P == 512)
     return a.d == 128 ? launch_fwd_t<128, 256, kPair>(a, W, sketch, lse, nullptr, st)
                       : launch_fwd_t<64, 256, kPair>(a, W, sketch, lse, nullptr, st);

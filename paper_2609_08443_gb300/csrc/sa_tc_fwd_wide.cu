@@ -1,54 +1,65 @@
-// Software-pipelined cluster-pair forward of the SA sketching step for
-// P = 512 prototypes (paper Sec. 3.1; FlashSA's streaming scheme, Sec. 4.4).
+// Cluster-pair forward of the SA sketching step for P = 512 prototypes with
+// sixteen softmax warps (paper Sec. 3.1; FlashSA's streaming scheme, Sec. 4.4).
 //
 // A cluster of two CTAs shares every 128-token tile; CTA r holds prototypes
-// [256 r, 256 r + 256), so each token's softmax over all 512 prototypes needs
-// the (max, sum) partials of four threads: the two warpgroups of each CTA,
-// each holding 128 of the token's scores.  The exchange crosses SMs and takes
-// longer than the rest of a tile's softmax, so the softmax warps overlap it
-// with the next tile:
+// [256 r, 256 r + 256).  The per-token softmax over all 512 prototypes is the
+// critical path of the step -- its exponentials alone keep an SM's MUFU busy
+// for a quarter of a tile's tensor time, and with two softmax warps per SM
+// sub-partition its dependent TMEM loads, max, exp, scale and stores left the
+// tensor pipe idle more than half the time.  Here four warpgroups share the
+// work: warpgroup g of CTA r holds, for every token of the tile, the 64 scores
+// of prototypes [256 r + 64 g, +64) -- four warps per sub-partition to hide
+// each other's latency, half the registers and instructions per thread.
 //
-//   A(i):  scores of tile i from TMEM (twice: max, then exp2 with that max),
-//          exponentials kept as fp16 pairs in registers, S released at once;
-//          the thread's (max, sum) goes to shared memory and, with st.async,
-//          into the peer CTA (four partials per token in each CTA).
-//   B(i-1): the four partials of tile i-1 (landed while A(i) ran) are combined
-//          in one fixed order -- bitwise the same (max, sum) in all four
-//          threads of a token --, the weights of tile i-1 are scaled and
-//          stored as bf16 for the aggregation UMMA.
-//
-// The UMMA issuer follows the same order: S(i+1) as soon as S(i) is released,
-// then O(i-1) once its weights are stored.  K and V tiles come from two
-// producers with rings of their own, so a V load held back by a pending
-// aggregation never delays the next K.
+// Per tile:
+//   1. TMA: K and V tiles from two producers with rings of their own; the
+//      prototype block Q ([256][d]) stays resident while the head does not
+//      change.
+//   2. UMMA  S^T = K Q^T  (M = 128 tokens, N = 256 prototypes, K = d) into TMEM.
+//   3. Each softmax thread loads its 64 scores, releases S at once, and forms
+//      exp2((s - m) c) with its own maximum m; its partial (m, sum) goes into
+//      this CTA's exchange buffer and, with st.async, into the peer CTA's, so
+//      both CTAs hold the eight partials of every token.  All four threads of
+//      a token in each CTA combine the eight in one fixed order: bitwise the
+//      same (max, sum) everywhere, and the per-token log-sum-exp.
+//   4. The weights, scaled by exp2((m - M) c) / Z, go to shared memory as bf16
+//      and UMMA accumulates the sketch: O^T += V^T A (d = 128) or O += A^T V.
+//   5. When a user's segment ends the sketch (or a worker's piece of it) is
+//      read back from TMEM and stored.
 // Warp roles: 0 = K producer (and prototypes), 1 = UMMA issuer, 2 = TMEM
-// allocator, 3 = V producer, 4..11 = softmax + epilogue.  Every wait is
+// allocator, 3 = V producer, 4..19 = softmax + epilogue.  Every wait is
 // bounded (sa_ptx.cuh).
 #include <cuda.h>
-#include <cuda_fp16.h>
 
 #include "sa_ptx.cuh"
 #include "sa_tc.cuh"
 #include "sa_tc_common.cuh"
 
 namespace sa {
-namespace tcp {
+namespace tcq {
 
 using namespace ptx;
 using namespace tcc;
 
-constexpr uint32_t kRegsCtl = 88, kRegsSoft = 208;
-static_assert(128 * kRegsCtl + 256 * kRegsSoft == 384 * 168, "register split = launch allocation");
+constexpr int kWThreads = 640;  // 20 warps
+constexpr int kWSoft0 = 4;      // warps 4..19: softmax / epilogue
+constexpr int kWSoftWarps = 16;
+// Registers: 640 threads launch with 96 each; the control warpgroup (producers,
+// issuer) keeps 64 and the four softmax warpgroups take 104.
+constexpr uint32_t kWRegsCtl = 64, kWRegsSoft = 104;
+static_assert(128 * kWRegsCtl + 512 * kWRegsSoft == 640 * 96, "register split = launch allocation");
 
 template <int D>
-struct PCfg {
-  static constexpr int PS = 256;  // prototypes per CTA
+struct WCfg {
+  static constexpr int PS = 256;    // prototypes per CTA
+  static constexpr int GP = 64;     // prototypes per softmax warpgroup
   static constexpr int KV_TILE = T * D * 2;
   static constexpr int Q_BYTES = PS * D * 2;
   static constexpr int W_BYTES = T * PS * 2;
   static constexpr int NK = (D == 128) ? 1 : 2;  // K slots
   static constexpr int NV = (D == 128) ? 1 : 2;  // V slots
-  static constexpr int X_BYTES = 2 * 4 * T * 8;  // [2 buffers][4 partials][T] (max, sum)
+  static constexpr int NPART = 8;                // partials per token: 4 warpgroups x 2 CTAs
+  static constexpr int X_BYTES = 2 * NPART * T * 8;  // [2 buffers][8 partials][T] (max, sum)
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + Q_BYTES;
   static constexpr int OFF_V = OFF_K + NK * KV_TILE;
@@ -62,32 +73,52 @@ struct PCfg {
   static constexpr int O_COLS = TRANS ? PS : (PS / 128) * D;
   static constexpr int S_COL = 0, O_COL = PS;
   static constexpr int TMEM_COLS = tmem_cols_for(PS + O_COLS);
-  static constexpr int HALF = PS / 2;  // prototypes per softmax warpgroup
   static_assert(SMEM <= 232448 && TMEM_COLS <= 512, "budget");
   static_assert(OFF_K % 1024 == 0 && OFF_V % 1024 == 0 && OFF_W % 1024 == 0, "swizzle atoms");
 };
 
-__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
-  const __half2 h = __floats2half2_rn(lo, hi);
-  return *reinterpret_cast<const uint32_t*>(&h);
-}
-__device__ __forceinline__ float2 unpack_f16(uint32_t w) {
-  return __half22float2(*reinterpret_cast<const __half2*>(&w));
+// The CTA's sketch block (256 prototypes x D) from TMEM to global memory,
+// shared by the 16 softmax warps: warp (g, q) takes TMEM lane quadrant q and
+// the g-th quarter of the columns.
+template <int D>
+__device__ __forceinline__ void store_block(uint32_t tmem, uint32_t lane_off, int g, int q, int lane, float* dst) {
+  using C = WCfg<D>;
+  float v[32];
+  if (C::TRANS) {  // lane = feature, column = prototype
+    const int d = 32 * q + lane;
+#pragma unroll 1
+    for (int c = 0; c < C::GP / 32; ++c) {
+      const int pbase = g * C::GP + 32 * c;
+      tmem_ld32(tmem + lane_off + C::O_COL + pbase, v);
+      tmem_ld_wait();
+      float* col = dst + int64_t(pbase) * D + d;
+#pragma unroll
+      for (int k = 0; k < 32; ++k) col[k * D] = v[k];
+    }
+  } else {  // two blocks of 128 prototypes on lanes, D = 64 columns each
+    const int blk = g >> 1, c = 32 * (g & 1);
+    const int p = 128 * blk + 32 * q + lane;
+    tmem_ld32(tmem + lane_off + C::O_COL + blk * D + c, v);
+    tmem_ld_wait();
+    float4* o = reinterpret_cast<float4*>(dst + int64_t(p) * D + c);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) o[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+  }
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    tc_fwd_pipe_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+__global__ void __launch_bounds__(kWThreads, 1)
+    tc_fwd_wide_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                        const __grid_constant__ CUtensorMap tmQ, Args a, float* __restrict__ sketch,
                        float* __restrict__ lse_out) {
-  using C = PCfg<D>;
+  using C = WCfg<D>;
   extern __shared__ __align__(1024) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // Both CTAs of a pair must reach the cluster barriers below, so a failed
   // call or a misaligned base only skips the work.
   bool skip = ws_failed(a.ws);
   if (smem_u32(smem) & 1023u) {
-    if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xA21u);
+    if (threadIdx.x == 0) ws_set_error(a.ws, SA_ERR_CUDA, 0xA31u);
     skip = true;
   }
   const uint32_t sbase = smem_u32(smem);
@@ -100,10 +131,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t b1 = bar0 + 8u * (2 * C::NK + 2 * C::NV);
   const uint32_t q_full = b1, q_empty = b1 + 8, s_full = b1 + 16, s_empty = b1 + 24, w_full = b1 + 32,
                  w_empty = b1 + 40, o_full = b1 + 48, o_empty = b1 + 56, drain = b1 + 64;
-  // exchange buffer b: x_full = the four partials are in (8 local warp arrivals
-  // + one arrival that expects the peer's 2 KB of st.async); x_free = this
-  // CTA's warps have read it; r_free = the PEER's warps have read theirs (so
-  // this CTA may push into it again)
+  // exchange buffer b (tiles alternate): x_full = the eight partials are in
+  // (16 local warp arrivals + one arrival expecting the peer's 4 KB of
+  // st.async); x_free = this CTA's warps have read it; r_free = the PEER's
+  // warps have read theirs, so this CTA may push into it again
   auto x_full = [&](int b) { return b1 + 72 + 8u * b; };
   auto x_free = [&](int b) { return b1 + 88 + 8u * b; };
   auto r_free = [&](int b) { return b1 + 104 + 8u * b; };
@@ -131,16 +162,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_full, 1);
     mbar_init(q_empty, 1);
     mbar_init(s_full, 1);
-    mbar_init(s_empty, kSoftWarps);
-    mbar_init(w_full, kSoftWarps);
+    mbar_init(s_empty, kWSoftWarps);
+    mbar_init(w_full, kWSoftWarps);
     mbar_init(w_empty, 1);
     mbar_init(o_full, 1);
-    mbar_init(o_empty, kSoftWarps);
+    mbar_init(o_empty, kWSoftWarps);
     mbar_init(drain, 1);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(x_full(b), kSoftWarps + 1);
-      mbar_init(x_free(b), kSoftWarps);
-      mbar_init(r_free(b), kSoftWarps);
+      mbar_init(x_full(b), kWSoftWarps + 1);
+      mbar_init(x_free(b), kWSoftWarps);
+      mbar_init(r_free(b), kWSoftWarps);
     }
     wait_ctl_init(abort_flag, a.ws);
     *skip_flag = skip ? 1u : 0u;
@@ -153,8 +184,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (ntiles > 0 && warp < kSoftWarp0) {
-    setmaxnreg_dec<kRegsCtl>();
+  if (ntiles > 0 && warp < kWSoft0) {
+    setmaxnreg_dec<kWRegsCtl>();
     if (warp == 0 && lane == 0) {
       // --------------------------------------------- K producer (+ prototypes)
       tma_prefetch_desc(&tmK);
@@ -175,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           pf.next();
         }
         if (it.qk != prev_q) {  // a new head (or, with per-user queries, a new user)
-          if (hc > 0) ok = mbar_wait(q_empty, uint32_t(hc - 1) & 1u, abort_flag, a.ws, 0x111);
+          if (hc > 0) ok = mbar_wait(q_empty, uint32_t(hc - 1) & 1u, abort_flag, a.ws, 0x121);
           if (!ok) break;
           mbar_arrive_expect_tx(q_full, C::Q_BYTES);
 #pragma unroll
@@ -184,7 +215,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++hc;
         }
         const int s = li % C::NK, use = li / C::NK;
-        if (use > 0) ok = mbar_wait(kempty(s), uint32_t(use - 1) & 1u, abort_flag, a.ws, 0x112);
+        if (use > 0) ok = mbar_wait(kempty(s), uint32_t(use - 1) & 1u, abort_flag, a.ws, 0x122);
         if (!ok) break;
         mbar_arrive_expect_tx(kfull(s), C::KV_TILE);
 #pragma unroll
@@ -205,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int li = 0; li < ntiles && ok; ++li) {
         const int s = li % C::NV, use = li / C::NV;
-        if (use > 0) ok = mbar_wait(vempty(s), uint32_t(use - 1) & 1u, abort_flag, a.ws, 0x113);
+        if (use > 0) ok = mbar_wait(vempty(s), uint32_t(use - 1) & 1u, abort_flag, a.ws, 0x123);
         if (!ok) break;
         mbar_arrive_expect_tx(vfull(s), C::KV_TILE);
 #pragma unroll
@@ -220,27 +251,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- UMMA issuer
-      // Order: S(0); then per tile i: S(i+1) once S(i) is released, O(i-1)
-      // once its weights are stored (the softmax warps' A(i+1) releases S(i+1)
-      // before their B(i) stores the weights of tile i).
+      // Order: S(0); then per tile i: S(i+1) once the softmax warps hold S(i)
+      // in registers, O(i) once the weights of tile i are stored.
       constexpr uint32_t idS = idesc_bf16(128, C::PS, 0, 0);
       constexpr uint32_t idO = C::TRANS ? idesc_bf16(128, C::PS, 1, 1) : idesc_bf16(128, D, 1, 1);
       TileWalker ws_(a, tb, te, T), wo(a, tb, te, T);
-      int hc = 0, sc = 0;
+      int hc = 0, sc = 0, prev_q = -1;
       bool ok = true;
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
       };
-      int prev_q = -1;
-      // S(li) = K(li) Q^T into the S columns; ws_ is at tile li
-      auto issue_S = [&](int li) {
+      auto issue_S = [&](int li) {  // ws_ is at tile li
         if (ws_.qk != prev_q) {
-          wt(q_full, uint32_t(hc) & 1u, 0x211);
+          wt(q_full, uint32_t(hc) & 1u, 0x221);
           ++hc;
           prev_q = ws_.qk;
         }
         const int s = li % C::NK;
-        wt(kfull(s), uint32_t(li / C::NK) & 1u, 0x212);
+        wt(kfull(s), uint32_t(li / C::NK) & 1u, 0x222);
         if (!ok) return;
         tc_fence_after();
         const uint32_t kaddr = sK + s * C::KV_TILE;
@@ -258,12 +286,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (li + 1 >= ntiles || qn != ws_.qk) umma_commit(q_empty);  // last S of these prototypes
         ws_.next();
       };
-      // O(li) += V(li)^T A(li) (or A^T V); wo is at tile li
-      auto issue_O = [&](int li) {
-        wt(w_full, uint32_t(li) & 1u, 0x213);
+      auto issue_O = [&](int li) {  // wo is at tile li
+        wt(w_full, uint32_t(li) & 1u, 0x223);
         const int s = li % C::NV;
-        wt(vfull(s), uint32_t(li / C::NV) & 1u, 0x214);
-        if (wo.seg_first && sc > 0) wt(o_empty, uint32_t(sc - 1) & 1u, 0x215);
+        wt(vfull(s), uint32_t(li / C::NV) & 1u, 0x224);
+        if (wo.seg_first && sc > 0) wt(o_empty, uint32_t(sc - 1) & 1u, 0x225);
         if (!ok) return;
         tc_fence_after();
         const uint32_t vaddr = sV + s * C::KV_TILE;
@@ -293,27 +320,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       issue_S(0);
       for (int li = 0; li < ntiles && ok; ++li) {
         if (li + 1 < ntiles) {
-          wt(s_empty, uint32_t(li) & 1u, 0x216);  // the softmax warps hold S(li)
+          wt(s_empty, uint32_t(li) & 1u, 0x226);  // the softmax warps hold S(li)
           if (ok) issue_S(li + 1);
         }
-        if (ok && li >= 1) issue_O(li - 1);
+        if (ok) issue_O(li);
       }
-      if (ok) issue_O(ntiles - 1);
       umma_commit(drain);  // no UMMA may still run when TMEM is released
       mbar_wait_bounded(drain, 0, 200000000ull);
     }
   } else if (ntiles > 0) {
-    setmaxnreg_inc<kRegsSoft>();
+    setmaxnreg_inc<kWRegsSoft>();
     // ------------------------------------------------ softmax + epilogue warps
-    const int sw = (warp - kSoftWarp0) >> 2;  // warpgroup: prototype half of this CTA
-    const int q = warp & 3;                   // TMEM lane quadrant
-    const int row = 32 * q + lane;            // token within the tile
+    const int g = (warp - kWSoft0) >> 2;  // warpgroup: prototypes [64 g, 64 g + 64) of this CTA
+    const int q = warp & 3;               // TMEM lane quadrant
+    const int row = 32 * q + lane;        // token within the tile
     const uint32_t lane_off = uint32_t(32 * q) << 16;
     const float c2 = a.scale * 1.4426950408889634f;  // scale * log2(e)
     float2* X = reinterpret_cast<float2*>(smem + C::OFF_X);
     const uint32_t x_peer = mapa_shared(sbase + C::OFF_X, peer);
-    const int slot = int(rank) * 2 + sw;  // this thread's partial among the four of its token
-    TileWalker wb(a, tb, te, T);  // the tile of phase B
+    const int slot = int(rank) * 4 + g;  // this thread's partial among the eight of its token
+    TileWalker cur(a, tb, te, T);
     bool ok = true;
     auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
       return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
@@ -321,136 +347,91 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto wwait_cl = [&](uint32_t bar, uint32_t par, uint32_t site) {
       return __all_sync(0xffffffffu, mbar_wait_cluster(bar, par, abort_flag, a.ws, site));
     };
-    uint32_t pk_prev[C::HALF / 2];  // exponentials of the previous tile, fp16 pairs
-    float m_prev = 0.f;
     int seg_idx = 0;
-    for (int it = 0; it <= ntiles && ok; ++it) {
-      uint32_t pk[C::HALF / 2];
-      float m = -INFINITY;
-      if (it < ntiles) {
-        // ------------------------------------------------------- A(it)
-        ok = wwait(s_full, uint32_t(it) & 1u, 0x311);
+    for (int li = 0; li < ntiles && ok; ++li) {
+      ok = wwait(s_full, uint32_t(li) & 1u, 0x321);
+      if (!ok) break;
+      tc_fence_after();
+      float v[C::GP];
+      tmem_ld32(tmem + lane_off + C::S_COL + g * C::GP, v);
+      tmem_ld32(tmem + lane_off + C::S_COL + g * C::GP + 32, v + 32);
+      tmem_ld_wait();
+      // S is in registers: its columns may take the next tile's scores
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(s_empty);
+      const float m = row_max<C::GP>(v);
+      const float z = exp2_shift_sum<C::GP>(v, c2, m * c2);
+      // this thread's partial into this CTA's exchange buffer and the peer's
+      const int b = li & 1;
+      if (li >= 2) {
+        ok = wwait(x_free(b), uint32_t((li - 2) >> 1) & 1u, 0x322);  // this CTA's readers of tile li-2
+        if (!ok) break;
+        ok = wwait_cl(r_free(b), uint32_t((li - 2) >> 1) & 1u, 0x323);  // the peer's readers of tile li-2
+        if (!ok) break;
+      }
+      const float2 part = make_float2(m, z);
+      X[(b * C::NPART + slot) * T + row] = part;
+      st_async_f2(x_peer + uint32_t(((b * C::NPART + slot) * T + row) * 8), part, mapa_shared(x_full(b), peer));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(x_full(b));
+      if (warp == kWSoft0 && lane == 0) mbar_arrive_expect_tx(x_full(b), 4u * T * 8u);
+      ok = wwait_cl(x_full(b), uint32_t(li >> 1) & 1u, 0x324);
+      if (!ok) break;
+      // the token's (max, sum) over all 512 prototypes, partials in slot order
+      float2 pp[C::NPART];
+#pragma unroll
+      for (int k = 0; k < C::NPART; ++k) pp[k] = X[(b * C::NPART + k) * T + row];
+      float M = pp[0].x;
+#pragma unroll
+      for (int k = 1; k < C::NPART; ++k) M = fmaxf(M, pp[k].x);
+      float Z = 0.f;
+#pragma unroll
+      for (int k = 0; k < C::NPART; ++k) Z = fmaf(pp[k].y, ex2((pp[k].x - M) * c2), Z);
+      // the partials are consumed (Z depends on every loaded value): the slots
+      // of this buffer may be rewritten, locally and by the peer
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(x_free(b));
+        mbar_arrive_relaxed_cluster(mapa_shared(r_free(b), peer));
+      }
+      const bool valid = row < cur.n;
+      // rows past the tile's tokens get exact zero weights
+      scale_row<C::GP>(v, valid ? ex2((m - M) * c2) / Z : 0.f);
+      if (rank == 0 && g == 0 && valid && lse_out) lse_out[(cur.tok0 + row) * a.H + cur.h] = M * a.scale + logf(Z);
+      if (li > 0) {
+        ok = wwait(w_empty, uint32_t(li - 1) & 1u, 0x325);  // O(li-1) has read the weights
+        if (!ok) break;
+      }
+      // weights -> shared memory, [PS/64 blocks][128 tokens][64 prototypes], 128-byte swizzle:
+      // warpgroup g fills block g
+      uint8_t* wrow = smem + C::OFF_W + g * (T * 128) + row * 128;
+#pragma unroll
+      for (int k = 0; k < C::GP / 8; ++k) {
+        uint4 pk;
+        pk.x = pack_bf16(v[8 * k + 0], v[8 * k + 1]);
+        pk.y = pack_bf16(v[8 * k + 2], v[8 * k + 3]);
+        pk.z = pack_bf16(v[8 * k + 4], v[8 * k + 5]);
+        pk.w = pack_bf16(v[8 * k + 6], v[8 * k + 7]);
+        *reinterpret_cast<uint4*>(wrow + ((k ^ (row & 7)) << 4)) = pk;
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(w_full);
+      if (cur.seg_last) {
+        ok = wwait(o_full, uint32_t(seg_idx) & 1u, 0x326);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t scol = tmem + lane_off + C::S_COL + sw * C::HALF;
-        {
-          float v[64];
-#pragma unroll
-          for (int c = 0; c < C::HALF / 64; ++c) {
-            tmem_ld32(scol + 64 * c, v);
-            tmem_ld32(scol + 64 * c + 32, v + 32);
-            tmem_ld_wait();
-            m = fmaxf(m, row_max<64>(v));
-          }
-        }
-        const float sh = m * c2;
-        float2 z0 = make_float2(0.f, 0.f), z1 = make_float2(0.f, 0.f);
-#pragma unroll
-        for (int c = 0; c < C::HALF / 32; ++c) {
-          float v[32];
-          tmem_ld32(scol + 32 * c, v);
-          tmem_ld_wait();
-          const float2 cc = make_float2(c2, c2), ns = make_float2(-sh, -sh);
-#pragma unroll
-          for (int j = 0; j < 32; j += 4) {
-            float2 x0 = __ffma2_rn(make_float2(v[j], v[j + 1]), cc, ns);
-            float2 x1 = __ffma2_rn(make_float2(v[j + 2], v[j + 3]), cc, ns);
-            x0.x = ex2(x0.x);
-            x0.y = ex2(x0.y);
-            x1.x = ex2(x1.x);
-            x1.y = ex2(x1.y);
-            z0 = __fadd2_rn(z0, x0);
-            z1 = __fadd2_rn(z1, x1);
-            pk[16 * c + j / 2] = pack_f16(x0.x, x0.y);
-            pk[16 * c + j / 2 + 1] = pack_f16(x1.x, x1.y);
-          }
-        }
-        const float z = (z0.x + z0.y) + (z1.x + z1.y);
-        // S(it) is in registers: its columns may take S(it+1)
+        const bool whole = cur.seg0 >= tb && cur.seg1 <= te;
+        float* dst = whole ? sketch + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D
+                           : a.partial + ((int64_t(wk) * 2 + partial_slot(total, W, wk, cur.seg0)) * a.P + p0) * D;
+        store_block<D>(tmem, lane_off, g, q, lane, dst);
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(s_empty);
-        // publish this thread's partial: into this CTA's buffer and the peer's
-        const int b = it & 1;
-        if (it >= 2) {
-          ok = wwait(x_free(b), uint32_t((it - 2) >> 1) & 1u, 0x312);  // this CTA's readers of tile it-2
-          if (!ok) break;
-        }
-        X[(b * 4 + slot) * T + row] = make_float2(m, z);
-        if (it >= 2) {
-          ok = wwait_cl(r_free(b), uint32_t((it - 2) >> 1) & 1u, 0x313);  // the peer's readers of tile it-2
-          if (!ok) break;
-        }
-        st_async_f2(x_peer + uint32_t(((b * 4 + slot) * T + row) * 8), make_float2(m, z),
-                    mapa_shared(x_full(b), peer));
-        __syncwarp();
-        if (lane == 0) mbar_arrive(x_full(b));
-        if (warp == kSoftWarp0 && lane == 0) mbar_arrive_expect_tx(x_full(b), 2u * T * 8u);
+        if (lane == 0) mbar_arrive(o_empty);
+        ++seg_idx;
       }
-      if (it >= 1) {
-        // ----------------------------------------------------- B(it - 1)
-        const int bp = (it - 1) & 1;
-        ok = wwait_cl(x_full(bp), uint32_t((it - 1) >> 1) & 1u, 0x314);
-        if (!ok) break;
-        const float2 p0v = X[(bp * 4 + 0) * T + row], p1v = X[(bp * 4 + 1) * T + row];
-        const float2 p2v = X[(bp * 4 + 2) * T + row], p3v = X[(bp * 4 + 3) * T + row];
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(x_free(bp));
-          mbar_arrive_cluster(mapa_shared(r_free(bp), peer));
-        }
-        // the token's (max, sum) over all 512 prototypes, in partial order 0..3
-        const float M = fmaxf(fmaxf(p0v.x, p1v.x), fmaxf(p2v.x, p3v.x));
-        const float Z = ((p0v.y * ex2((p0v.x - M) * c2) + p1v.y * ex2((p1v.x - M) * c2)) +
-                         p2v.y * ex2((p2v.x - M) * c2)) +
-                        p3v.y * ex2((p3v.x - M) * c2);
-        const bool valid = row < wb.n;
-        // rows past the tile's tokens get exact zero weights
-        const float f = valid ? ex2((m_prev - M) * c2) / Z : 0.f;
-        if (rank == 0 && sw == 0 && valid && lse_out) lse_out[(wb.tok0 + row) * a.H + wb.h] = M * a.scale + logf(Z);
-        if (it >= 2) {
-          ok = wwait(w_empty, uint32_t(it - 2) & 1u, 0x315);  // O(it-2) has read the weights
-          if (!ok) break;
-        }
-        // weights -> shared memory, [PS/64 blocks][128 tokens][64 prototypes], 128-byte swizzle
-        uint8_t* wrow = smem + C::OFF_W + row * 128;
-        const float2 ff = make_float2(f, f);
-#pragma unroll
-        for (int k = 0; k < C::HALF / 8; ++k) {
-          const int p = sw * C::HALF + 8 * k;
-          const int blk = p >> 6, chunk = (p & 63) >> 3;
-          uint32_t o[4];
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const float2 e = __fmul2_rn(unpack_f16(pk_prev[4 * k + j]), ff);
-            o[j] = pack_bf16(e.x, e.y);
-          }
-          *reinterpret_cast<uint4*>(wrow + blk * (T * 128) + ((chunk ^ (row & 7)) << 4)) =
-              make_uint4(o[0], o[1], o[2], o[3]);
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(w_full);
-        if (wb.seg_last) {
-          ok = wwait(o_full, uint32_t(seg_idx) & 1u, 0x316);
-          if (!ok) break;
-          tc_fence_after();
-          const bool whole = wb.seg0 >= tb && wb.seg1 <= te;
-          float* dst = whole ? sketch + ((int64_t(wb.b) * a.H + wb.h) * a.P + p0) * D
-                             : a.partial + ((int64_t(wk) * 2 + partial_slot(total, W, wk, wb.seg0)) * a.P + p0) * D;
-          store_sketch<D, C::PS, C::TRANS, C::O_COL>(tmem, lane_off, sw, q, lane, dst);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(o_empty);
-          ++seg_idx;
-        }
-        wb.next();
-      }
-      if (it < ntiles) {
-#pragma unroll
-        for (int j = 0; j < C::HALF / 2; ++j) pk_prev[j] = pk[j];
-        m_prev = m;
-      }
+      cur.next();
     }
   }
   __syncthreads();
@@ -463,19 +444,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int D>
-static cudaError_t launch_pipe_t(const Args& a, int W, float* sketch, float* lse_out, cudaStream_t st) {
-  using C = PCfg<D>;
+static cudaError_t launch_wide_t(const Args& a, int W, float* sketch, float* lse_out, cudaStream_t st) {
+  using C = WCfg<D>;
   CUtensorMap tk, tv, tq;
   if (!make_kv_map(&tk, a.K, a.N, a.H, D) || !make_kv_map(&tv, a.V, a.N, a.H, D) ||
       !make_q_map(&tq, a.Q, a.uq ? a.B * a.H : a.H, a.P, D, C::PS))
     return cudaErrorInvalidValue;
-  auto fn = &tc_fwd_pipe_kernel<D>;
+  auto fn = &tc_fwd_wide_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   // one cluster of two CTAs per worker; CTA rank r holds prototypes [256 r, 256 r + 256)
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * W, 1, 1);
-  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.blockDim = dim3(kWThreads, 1, 1);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
@@ -488,11 +469,11 @@ static cudaError_t launch_pipe_t(const Args& a, int W, float* sketch, float* lse
   return cudaLaunchKernelEx(&cfg, fn, tk, tv, tq, a, sketch, lse_out);
 }
 
-}  // namespace tcp
+}  // namespace tcq
 
-cudaError_t launch_tc_fwd_pipe(const Args& a, int W, float* sketch, float* lse, cudaStream_t st) {
+cudaError_t launch_tc_fwd_wide(const Args& a, int W, float* sketch, float* lse, cudaStream_t st) {
   if (a.N == 0) return cudaSuccess;
-  return a.d == 128 ? tcp::launch_pipe_t<128>(a, W, sketch, lse, st) : tcp::launch_pipe_t<64>(a, W, sketch, lse, st);
+  return a.d == 128 ? tcq::launch_wide_t<128>(a, W, sketch, lse, st) : tcq::launch_wide_t<64>(a, W, sketch, lse, st);
 }
 
 }  // namespace sa

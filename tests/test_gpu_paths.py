@@ -53,15 +53,16 @@ def test_pair_forward_matches_lse_pass_and_slices(cuda_lib, P, d):
 
 
 @pytest.mark.parametrize("P,d", [(512, 128), (512, 64)])
-def test_pipelined_pair_forward_matches_unpipelined(cuda_lib, P, d):
-    """The software-pipelined cluster-pair forward (tile i's (max, sum) exchange
-    overlapped with tile i+1's scores) against the same pair split without the
-    pipeline, on ragged users that end tiles, segments and worker ranges at
-    every offset; the pipelined kernel is also bitwise reproducible."""
+def test_wide_pair_forward_matches_narrow(cuda_lib, P, d):
+    """The cluster-pair forward with sixteen softmax warps per CTA (eight
+    partial (max, sum) per token) against the pair kernel with eight softmax
+    warps (four partials), on ragged users that end tiles, segments and worker
+    ranges at every offset; the sixteen-warp kernel is also bitwise
+    reproducible."""
     spec = wl.custom([700, 0, 128, 129, 3000, 1, 5000, 2, 255, 257], H=3, P=P, d=d, dtype=wl.BF16, seed=P + d + 1)
     host = wl.make_host(spec)
     t = wl.host_to_torch(spec, host, torch.device("cuda"))
-    assert "pipe" in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
+    assert "wide" in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
     pipe = harness.gpu_outputs(spec, t, bwd=False)
     pipe2 = harness.gpu_outputs(spec, t, bwd=False)
     binding.sa_select_path(3)
