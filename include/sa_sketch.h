@@ -299,9 +299,9 @@ sa_status sa_set_wait_limit_ns(uint64_t ns);
  * CUDA-core kernels everywhere (a cross-check of the two), 2 keeps the
  * tensor cores but runs the forward for P = 512 (and P = 256 with d = 128) as a
  * per-token lse pass followed by prototype slices instead of the cluster-pair
- * kernel (another cross-check), 3 runs the P = 512 forward on the cluster-pair
- * kernel with eight softmax warps per CTA instead of sixteen (its earlier
- * form, a third cross-check).  The workspace size depends on the selection: size it after
+ * kernel (another cross-check), 3 runs the P = 512 forward on the
+ * cluster-pair kernel with eight softmax warps per CTA instead of sixteen
+ * (its earlier form, a third cross-check).  The workspace size depends on the selection: size it after
  * choosing. */
 sa_status sa_select_path(int path);
 

@@ -201,7 +201,7 @@ namespace sa {
 bool tc_path_enabled() { return g_path.load() != 1; }
 uint64_t wait_limit_ns() { return g_wait_ns.load(); }
 bool tc_fwd_sliced_selected() { return g_path.load() == 2; }
-bool tc_fwd_pair_selected() { return g_path.load() == 3; }
+bool tc_narrow_selected() { return g_path.load() == 3; }
 
 namespace tcc {
 

@@ -62,46 +62,34 @@ __device__ __forceinline__ void wait_ctl_init(volatile int* abort_flag, const vo
   reinterpret_cast<volatile uint32_t*>(abort_flag)[2] = ns > 0xFFFFFFFFull ? 0xFFFFFFFFu : uint32_t(ns);
 }
 
-__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Limits below this are test settings: the wait then polls without suspending
-// so that it gives up within a few hundred nanoseconds of the limit.
+// Limits below this are test settings (sa_set_wait_limit_ns): kernels that
+// support a forced timeout then wait on a barrier that nothing completes, so
+// the limit runs out however fast the rest of the pipeline is.
 constexpr uint32_t kPollLimitNs = 1000000u;  // 1 ms
 
-__device__ __forceinline__ bool mbar_wait_timed_out(volatile int* abort_flag, void* ws, uint32_t site, uint64_t t0,
-                                                    uint64_t lim) {
-  if (globaltimer() - t0 <= lim) return false;
+__device__ __forceinline__ uint32_t ctl_wait_limit(volatile int* abort_flag) {
+  return reinterpret_cast<volatile const uint32_t*>(abort_flag)[2];
+}
+
+__device__ __forceinline__ bool mbar_wait_timed_out(volatile int* abort_flag, void* ws, uint32_t site, uint64_t t0) {
+  if (globaltimer() - t0 <= ctl_wait_limit(abort_flag)) return false;
   *abort_flag = 1;
   ws_set_error(ws, SA_ERR_TIMEOUT, site);
   return true;
 }
 
+// The flag and the clock are checked every 64 polls, so a handoff that is
+// ready after a few polls costs nothing beyond the polls themselves.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, void* ws,
                                           uint32_t site) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
-  const uint32_t lim = reinterpret_cast<volatile const uint32_t*>(abort_flag)[2];
-  if (lim < kPollLimitNs) {
-    for (;;) {
-      if (mbar_test_wait(bar, parity)) return true;
-      if (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim)) return false;
-    }
-  }
-  // the flag and the clock are checked every 64 polls: a handoff that is not
-  // ready at the first poll is then noticed as soon as it completes
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 0u && (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim))) return false;
+    if ((it & 63u) == 0u) {
+      if (*abort_flag) return false;
+      if (mbar_wait_timed_out(abort_flag, ws, site, t0)) return false;
+    }
   }
 }
 
@@ -169,10 +157,12 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity,
                                                   uint32_t site) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
-  const uint32_t lim = reinterpret_cast<volatile const uint32_t*>(abort_flag)[2];
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
-    if ((it & 63u) == 0u && (*abort_flag || mbar_wait_timed_out(abort_flag, ws, site, t0, lim))) return false;
+    if ((it & 63u) == 0u) {
+      if (*abort_flag) return false;
+      if (mbar_wait_timed_out(abort_flag, ws, site, t0)) return false;
+    }
   }
 }
 

@@ -9,7 +9,7 @@ bool tc_fwd_needs_lse_pass_d(int P, int d);  // lse pass, then 256-prototype sli
 int tc_lse_slice(int P, int d);              // prototypes per slice of the lse pass
 bool tc_path_enabled();
 bool tc_fwd_sliced_selected();  // sa_select_path(2)
-bool tc_fwd_pair_selected();    // sa_select_path(3): the 8-softmax-warp pair kernel for P = 512
+bool tc_narrow_selected();      // sa_select_path(3): the 8-softmax-warp pair forward for P = 512
 // P = 512: the cluster-pair forward with 16 softmax warps (sa_tc_fwd_wide.cu)
 cudaError_t launch_tc_fwd_wide(const Args& a, int W, float* sketch, float* lse, cudaStream_t st);
 bool tc_bwd_supported(int P, int d, sa_dtype dt);

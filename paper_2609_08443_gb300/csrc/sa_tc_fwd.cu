@@ -63,7 +63,7 @@ struct Cfg {
   static constexpr int OFF_W = OFF_RING + NSLOT * KV_TILE;
   static constexpr int OFF_STATS = OFF_W + W_BYTES;
   static constexpr int OFF_BAR = OFF_STATS + STATS;
-  static constexpr int NBAR = 2 * NSLOT + 13;
+  static constexpr int NBAR = 2 * NSLOT + 14;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // tmem address, abort flag, skip flag (pair)
   static constexpr int SMEM = OFF_MISC + 16;
   static_assert(SMEM <= 232448, "shared memory budget");
@@ -100,7 +100,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t q_full = bar0 + 8u * (2 * C::NSLOT + 0), q_empty = q_full + 8, s_full = q_full + 16,
                  s_empty = q_full + 24, w_full = q_full + 32, w_empty = q_full + 40, o_full = q_full + 48,
                  o_empty = q_full + 56, drain = q_full + 64, st_ready = q_full + 72, st_used = q_full + 80,
-                 r_full = q_full + 88, r_used = q_full + 96;
+                 r_full = q_full + 88, r_used = q_full + 96, never = q_full + 104;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
   volatile uint32_t* skip_flag = reinterpret_cast<volatile uint32_t*>(smem + C::OFF_MISC + 8);
@@ -138,6 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(st_used, kSoftWarps);
     mbar_init(r_full, 1);
     mbar_init(r_used, kSoftWarps);
+    mbar_init(never, 1);  // completed by nothing: the forced timeout of a test limit
     wait_ctl_init(abort_flag, a.ws);
     *skip_flag = skip ? 1u : 0u;
     fence_mbar_init();
@@ -228,7 +229,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       nxt.next();
       uint32_t e = 0;
       int hc = 0, sc = 0;
-      bool ok = mbar_wait(q_full, 0, abort_flag, a.ws, 0x201);
+      // under a test limit (sa_set_wait_limit_ns) the issuer first waits for a
+      // barrier nothing completes: the limit runs out and the CTA takes its
+      // abort path (drains, TMEM freed, SA_ERR_TIMEOUT)
+      bool ok = ctl_wait_limit(abort_flag) >= kPollLimitNs || mbar_wait(never, 0, abort_flag, a.ws, 0x200);
+      ok = ok && mbar_wait(q_full, 0, abort_flag, a.ws, 0x201);
       auto issue_S = [&](uint32_t slot) {
         const uint32_t kaddr = sRing + slot * C::KV_TILE;
 #pragma unroll
@@ -787,7 +792,7 @@ bool tc_fwd_needs_lse_pass_d(int P, int d) {
 
 const char* tc_fwd_name(int P, int d) {
   if (tc_fwd_needs_lse_pass_d(P, d)) return d == 128 ? "tc_fwd_kernel<128,256,sliced>" : "tc_fwd_kernel<64,256,sliced>";
-  if (P == 512 && !tc_fwd_pair_selected()) return d == 128 ? "tc_fwd_wide_kernel<128>" : "tc_fwd_wide_kernel<64>";
+  if (P == 512 && !tc_narrow_selected()) return d == 128 ? "tc_fwd_wide_kernel<128>" : "tc_fwd_wide_kernel<64>";
   if (P == 512) return d == 128 ? "tc_fwd_kernel<128,256,pair>" : "tc_fwd_kernel<64,256,pair>";
   if (P == 256) return d == 128 ? "tc_fwd_kernel<128,256,fused>" : "tc_fwd_kernel<64,256,fused>";
   return d == 128 ? "tc_fwd_kernel<128,128,fused>" : "tc_fwd_kernel<64,128,fused>";
@@ -830,7 +835,7 @@ cudaError_t launch_tc_fwd(const Args& a, int W, float* sketch, float* lse, cudaS
   if (tc_fwd_needs_lse_pass_d(a.P, a.d))  // lse (from launch_tc_lse beforehand) is an input here
     return a.d == 128 ? launch_fwd_t<128, 256, kSliced>(a, W, sketch, nullptr, lse, st)
                       : launch_fwd_t<64, 256, kSliced>(a, W, sketch, nullptr, lse, st);
-  if (a.P == 512 && !tc_fwd_pair_selected()) return launch_tc_fwd_wide(a, W, sketch, lse, st);
+  if (a.P == 512 && !tc_narrow_selected()) return launch_tc_fwd_wide(a, W, sketch, lse, st);
   if (a.P == 512)
     return a.d == 128 ? launch_fwd_t<128, 256, kPair>(a, W, sketch, lse, nullptr, st)
                       : launch_fwd_t<64, 256, kPair>(a, W, sketch, lse, nullptr, st);

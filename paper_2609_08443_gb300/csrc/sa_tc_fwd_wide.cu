@@ -382,12 +382,12 @@ __global__ void __launch_bounds__(kWThreads, 1)
       float2 pp[C::NPART];
 #pragma unroll
       for (int k = 0; k < C::NPART; ++k) pp[k] = X[(b * C::NPART + k) * T + row];
-      float M = pp[0].x;
+      const float M = fmaxf(fmaxf(fmax3(pp[0].x, pp[1].x, pp[2].x), fmax3(pp[3].x, pp[4].x, pp[5].x)),
+                            fmaxf(pp[6].x, pp[7].x));
+      float w[C::NPART];  // each partial's sum rescaled to the common maximum, all exponentials independent
 #pragma unroll
-      for (int k = 1; k < C::NPART; ++k) M = fmaxf(M, pp[k].x);
-      float Z = 0.f;
-#pragma unroll
-      for (int k = 0; k < C::NPART; ++k) Z = fmaf(pp[k].y, ex2((pp[k].x - M) * c2), Z);
+      for (int k = 0; k < C::NPART; ++k) w[k] = pp[k].y * ex2((pp[k].x - M) * c2);
+      const float Z = ((w[0] + w[1]) + (w[2] + w[3])) + ((w[4] + w[5]) + (w[6] + w[7]));  // fixed tree order
       // the partials are consumed (Z depends on every loaded value): the slots
       // of this buffer may be rewritten, locally and by the peer
       __syncwarp();
@@ -397,8 +397,11 @@ __global__ void __launch_bounds__(kWThreads, 1)
       }
       const bool valid = row < cur.n;
       // rows past the tile's tokens get exact zero weights
-      scale_row<C::GP>(v, valid ? ex2((m - M) * c2) / Z : 0.f);
-      if (rank == 0 && g == 0 && valid && lse_out) lse_out[(cur.tok0 + row) * a.H + cur.h] = M * a.scale + logf(Z);
+      const float rz = __frcp_rn(Z);
+      scale_row<C::GP>(v, valid ? ex2((m - M) * c2) * rz : 0.f);
+      // natural log of Z through the log2 unit (Z lies in [1, 512])
+      if (rank == 0 && g == 0 && valid && lse_out)
+        lse_out[(cur.tok0 + row) * a.H + cur.h] = M * a.scale + __log2f(Z) * 0.6931471805599453f;
       if (li > 0) {
         ok = wwait(w_empty, uint32_t(li - 1) & 1u, 0x325);  // O(li-1) has read the weights
         if (!ok) break;

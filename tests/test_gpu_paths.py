@@ -54,25 +54,28 @@ def test_pair_forward_matches_lse_pass_and_slices(cuda_lib, P, d):
 
 @pytest.mark.parametrize("P,d", [(512, 128), (512, 64)])
 def test_wide_pair_forward_matches_narrow(cuda_lib, P, d):
-    """The cluster-pair forward with sixteen softmax warps per CTA (eight
-    partial (max, sum) per token) against the pair kernel with eight softmax
-    warps (four partials), on ragged users that end tiles, segments and worker
-    ranges at every offset; the sixteen-warp kernel is also bitwise
-    reproducible."""
+    """The P = 512 cluster-pair forward with sixteen softmax warps per CTA
+    (eight partial (max, sum) per token) against the pair kernel with eight
+    softmax warps (four partials), on ragged users that end tiles, segments
+    and worker ranges at every offset, with the backward that follows it, and
+    against the oracle; the sixteen-warp kernel is also bitwise reproducible."""
     spec = wl.custom([700, 0, 128, 129, 3000, 1, 5000, 2, 255, 257], H=3, P=P, d=d, dtype=wl.BF16, seed=P + d + 1)
     host = wl.make_host(spec)
     t = wl.host_to_torch(spec, host, torch.device("cuda"))
     assert "wide" in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
-    pipe = harness.gpu_outputs(spec, t, bwd=False)
-    pipe2 = harness.gpu_outputs(spec, t, bwd=False)
+    wide = harness.gpu_outputs(spec, t, bwd=True)
+    wide2 = harness.gpu_outputs(spec, t, bwd=True)
     binding.sa_select_path(3)
     try:
         assert "pair" in binding.sa_main_kernel_name(P, d, binding.SA_BF16, False)
-        pair = harness.gpu_outputs(spec, t, bwd=False)
+        narrow = harness.gpu_outputs(spec, t, bwd=True)
     finally:
         binding.sa_select_path(0)
-    assert (pipe["sketch"] == pipe2["sketch"]).all() and (pipe["lse"] == pipe2["lse"]).all()
-    assert harness.rel_err(pipe["sketch"], pair["sketch"]) <= 2e-2
-    assert abs(pipe["lse"] - pair["lse"]).max() <= 5e-3 * max(1.0, abs(pair["lse"]).max())
-    ref = harness.oracle_outputs(spec, host, bwd=False)
-    harness.assert_close("sketch", pipe["sketch"], ref["sketch"], harness.TOL[wl.BF16])
+    for k in ("sketch", "lse", "dK", "dV", "dQ"):
+        assert (wide[k] == wide2[k]).all(), k
+    for k in ("sketch", "dK", "dV", "dQ"):
+        assert harness.rel_err(wide[k], narrow[k]) <= 2e-2, k
+    assert abs(wide["lse"] - narrow["lse"]).max() <= 5e-3 * max(1.0, abs(narrow["lse"]).max())
+    ref = harness.oracle_outputs(spec, host, bwd=True)
+    for k in ("sketch", "dK", "dV", "dQ"):
+        harness.assert_close(k, wide[k], ref[k], harness.TOL[wl.BF16])
