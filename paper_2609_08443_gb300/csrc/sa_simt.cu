@@ -71,12 +71,48 @@ __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ 
   }
 }
 
+// out[e] (+)= sum over k < n of src[off[k] + e] for e < PD, in k order; the
+// first chunk of workers starts from zero, later chunks continue the running
+// sum held in out (so the rounding is that of one sum in worker order).  A
+// negative off[k] is a worker with an empty range.  float4 accesses when every
+// address is 16-byte aligned.
+__device__ __forceinline__ void sum_pieces(const float* __restrict__ src, const int64_t* off, int n,
+                                           bool first, int64_t PD, float* __restrict__ out, int64_t e0,
+                                           int64_t estep) {
+  bool vec = (PD & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(out)) & 15) == 0;
+  if (vec) {
+    const float4* s4 = reinterpret_cast<const float4*>(src);
+    float4* o4 = reinterpret_cast<float4*>(out);
+    for (int64_t e = e0; e < PD / 4; e += estep) {
+      float4 s = first ? make_float4(0.f, 0.f, 0.f, 0.f) : o4[e];
+      for (int k = 0; k < n; ++k) {
+        if (off[k] < 0) continue;
+        const float4 v = s4[off[k] / 4 + e];
+        s.x += v.x;
+        s.y += v.y;
+        s.z += v.z;
+        s.w += v.w;
+      }
+      o4[e] = s;
+    }
+    return;
+  }
+  for (int64_t e = e0; e < PD; e += estep) {
+    float s = first ? 0.f : out[e];
+    for (int k = 0; k < n; ++k)
+      if (off[k] >= 0) s += src[off[k] + e];
+    out[e] = s;
+  }
+}
+
 // Sum of the pieces of every cut (user, head) segment, in worker order; zero
-// sketch for empty users.  grid = B*H blocks.
+// sketch for empty users.  grid = B*H blocks.  The pieces' offsets are found
+// once per block (range_begin divides in 64 bits), then summed element-wise.
 __global__ void __launch_bounds__(256) finalize_sketch_kernel(const void* ws, const int64_t* prefix,
                                                               int B, int H, int P, int d, int W,
                                                               const float* __restrict__ partial,
                                                               float* __restrict__ sketch) {
+  __shared__ int64_t off[256];
   if (ws_failed(ws)) return;
   const int64_t tph = reinterpret_cast<const WsHeader*>(ws)->tiles_per_head;
   const int64_t total = tph * H;
@@ -90,14 +126,17 @@ __global__ void __launch_bounds__(256) finalize_sketch_kernel(const void* ws, co
   }
   const int g0 = owner_of(total, W, seg0), g1 = owner_of(total, W, seg1 - 1);
   if (g0 == g1) return;  // written whole by its worker
-  for (int64_t e = threadIdx.x; e < PD; e += blockDim.x) {
-    float s = 0.f;
-    for (int g = g0; g <= g1; ++g) {
-      if (range_begin(total, W, g) == range_begin(total, W, g + 1)) continue;
-      const int slot = partial_slot(total, W, g, seg0);
-      s += partial[(int64_t(g) * 2 + slot) * PD + e];
+  for (int c0 = g0; c0 <= g1; c0 += 256) {
+    const int n = min(256, g1 - c0 + 1);
+    __syncthreads();
+    if (int(threadIdx.x) < n) {
+      const int g = c0 + int(threadIdx.x);
+      off[threadIdx.x] = range_begin(total, W, g) == range_begin(total, W, g + 1)
+                             ? int64_t(-1)
+                             : (int64_t(g) * 2 + partial_slot(total, W, g, seg0)) * PD;
     }
-    out[e] = s;
+    __syncthreads();
+    sum_pieces(partial, off, n, c0 == g0, PD, out, threadIdx.x, blockDim.x);
   }
 }
 
@@ -105,25 +144,30 @@ __global__ void __launch_bounds__(256) finalize_sketch_kernel(const void* ws, co
 __global__ void __launch_bounds__(256) finalize_dq_kernel(const void* ws, int H, int P, int d, int W,
                                                           const float* __restrict__ dq_partial,
                                                           float* __restrict__ dQ) {
+  __shared__ int64_t off[256];
   if (ws_failed(ws)) return;
   const int64_t tph = reinterpret_cast<const WsHeader*>(ws)->tiles_per_head;
   const int64_t total = tph * H;
   const int h = blockIdx.y;
   const int64_t PD = int64_t(P) * d;
   float* out = dQ + int64_t(h) * PD;
-  const int64_t stride = int64_t(gridDim.x) * blockDim.x;
+  const int64_t e0 = blockIdx.x * int64_t(blockDim.x) + threadIdx.x, stride = int64_t(gridDim.x) * blockDim.x;
   if (tph == 0) {
-    for (int64_t e = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; e < PD; e += stride) out[e] = 0.f;
+    for (int64_t e = e0; e < PD; e += stride) out[e] = 0.f;
     return;
   }
   const int g0 = owner_of(total, W, int64_t(h) * tph), g1 = owner_of(total, W, int64_t(h + 1) * tph - 1);
-  for (int64_t e = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; e < PD; e += stride) {
-    float s = 0.f;
-    for (int g = g0; g <= g1; ++g) {
-      if (range_begin(total, W, g) == range_begin(total, W, g + 1)) continue;
-      s += dq_partial[(int64_t(g) * H + h) * PD + e];
+  for (int c0 = g0; c0 <= g1; c0 += 256) {
+    const int n = min(256, g1 - c0 + 1);
+    __syncthreads();
+    if (int(threadIdx.x) < n) {
+      const int g = c0 + int(threadIdx.x);
+      off[threadIdx.x] = range_begin(total, W, g) == range_begin(total, W, g + 1)
+                             ? int64_t(-1)
+                             : (int64_t(g) * H + h) * PD;
     }
-    out[e] = s;
+    __syncthreads();
+    sum_pieces(dq_partial, off, n, c0 == g0, PD, out, e0, stride);
   }
 }
 
