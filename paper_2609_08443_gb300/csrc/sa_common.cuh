@@ -107,6 +107,7 @@ struct TileRef {
   int n;          // tokens in the tile (1..T)
   int64_t seg0;   // global index of the segment's first tile
   int64_t seg1;   // one past the segment's last tile
+  int64_t L;      // the user's tokens
 };
 
 SA_HD TileRef locate_tile(int64_t t, int64_t tph, const int64_t* prefix, const int32_t* cu,
@@ -118,10 +119,40 @@ SA_HD TileRef locate_tile(int64_t t, int64_t tph, const int64_t* prefix, const i
   int64_t k = rem - prefix[r.b];
   int64_t L = int64_t(cu[r.b + 1]) - int64_t(cu[r.b]);
   r.tok0 = int64_t(cu[r.b]) + k * T;
+  r.L = L;
   int64_t left = L - k * T;
   r.n = int(left < T ? left : T);
   r.seg0 = int64_t(r.h) * tph + prefix[r.b];
   r.seg1 = int64_t(r.h) * tph + prefix[r.b + 1];
+  return r;
+}
+
+// locate_tile for tile t, the first tile of the segment that follows segment
+// (h_prev, b_prev) in the tile order.  The user is found by a short forward
+// scan from b_prev + 1 (or from 0 in a new head) instead of a binary search:
+// consecutive segments are consecutive non-empty users, so the scan usually
+// takes one step.  The answer is accepted only where it meets find_user's
+// definition (prefix[b] <= r < prefix[b + 1]); a long run of empty users
+// falls back to the search.
+SA_HD TileRef locate_next_segment(int64_t t, int h_prev, int b_prev, int64_t tph, const int64_t* prefix,
+                                  const int32_t* cu, int B, int T) {
+  const int h = int(t / tph);
+  const int64_t rem = t - int64_t(h) * tph;
+  int c = h == h_prev ? b_prev + 1 : 0;
+  if (c >= B) c = B - 1;
+  for (int steps = 0; steps < 8 && c + 1 < B && prefix[c + 1] <= rem; ++steps) ++c;
+  if (!(prefix[c] <= rem && (c + 1 >= B || prefix[c + 1] > rem))) return locate_tile(t, tph, prefix, cu, B, T);
+  TileRef r;
+  r.h = h;
+  r.b = c;
+  const int64_t k = rem - prefix[c];
+  const int64_t cb = int64_t(cu[c]), L = int64_t(cu[c + 1]) - cb;
+  r.tok0 = cb + k * T;
+  r.L = L;
+  const int64_t left = L - k * T;
+  r.n = int(left < T ? left : T);
+  r.seg0 = int64_t(h) * tph + prefix[c];
+  r.seg1 = int64_t(h) * tph + prefix[c + 1];
   return r;
 }
 

@@ -1533,7 +1533,7 @@ __device__ __forceinline__ void bwd_dq_body(const CUtensorMap& tmK, const CUtens
         // the next tile opens a new (user, head) segment: its dsketch slice goes in
         // before S and dA of that tile are issued (they wait for sda_free and g_full)
         if (li + 1 < ntiles && cur.seg_last) {
-          const TileRef nx = locate_tile(cur.t + 1, cur.tph, a.prefix, a.cu, a.B, T);
+          const TileRef nx = locate_next_segment(cur.t + 1, cur.h, cur.b, cur.tph, a.prefix, a.cu, a.B, T);
           if (!put_g(nx.b, nx.h)) {
             ok = false;
             break;

@@ -38,8 +38,8 @@ struct TileWalker {
     tph = reinterpret_cast<const WsHeader*>(a.ws)->tiles_per_head;
     if (t < te) relocate();
   }
-  __device__ void relocate() {
-    const TileRef r = locate_tile(t, tph, prefix, cu, B, Tt);
+  __device__ void relocate() { set(locate_tile(t, tph, prefix, cu, B, Tt)); }
+  __device__ void set(const TileRef& r) {
     h = r.h;
     b = r.b;
     qk = uq ? b * H + h : h;
@@ -47,8 +47,8 @@ struct TileWalker {
     seg1 = r.seg1;
     nk = seg1 - seg0;
     k = t - seg0;
-    cub = int64_t(cu[b]);
-    Lb = int64_t(cu[b + 1]) - cub;
+    cub = r.tok0 - k * Tt;
+    Lb = r.L;
     fields();
   }
   __device__ void fields() {
@@ -79,7 +79,7 @@ struct TileWalker {
       h_n = h;
       qk_n = qk;
     } else {
-      const TileRef r = locate_tile(t + 1, tph, prefix, cu, B, Tt);
+      const TileRef r = locate_next_segment(t + 1, h, b, tph, prefix, cu, B, Tt);
       tok0_n = r.tok0;
       n_n = r.n;
       h_n = r.h;
@@ -93,7 +93,7 @@ struct TileWalker {
       ++k;
       fields();
     } else {
-      relocate();
+      set(locate_next_segment(t, h, b, tph, prefix, cu, B, Tt));
     }
   }
 };

@@ -63,7 +63,7 @@ struct Cfg {
   static constexpr int OFF_W = OFF_RING + NSLOT * KV_TILE;
   static constexpr int OFF_STATS = OFF_W + W_BYTES;
   static constexpr int OFF_BAR = OFF_STATS + STATS;
-  static constexpr int NBAR = 2 * NSLOT + 14;
+  static constexpr int NBAR = 2 * NSLOT + 16;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // tmem address, abort flag, skip flag (pair)
   static constexpr int SMEM = OFF_MISC + 16;
   static_assert(SMEM <= 232448, "shared memory budget");
@@ -71,7 +71,10 @@ struct Cfg {
   static constexpr int O_COLS = TRANS ? PS : (PS / 128) * D;
   static constexpr int S_COL = 0;
   static constexpr int O_COL = PS;
-  static constexpr int TMEM_COLS = tmem_cols_for(PS + O_COLS);
+  // two sketch accumulators where TMEM holds them: a segment's sketch is stored
+  // while the next segment accumulates into the other one
+  static constexpr int NOB = (PS + 2 * O_COLS <= 512) ? 2 : 1;
+  static constexpr int TMEM_COLS = tmem_cols_for(PS + NOB * O_COLS);
   static constexpr int HALF = PS / 2;  // prototypes per softmax warpgroup
 };
 
@@ -101,6 +104,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                  s_empty = q_full + 24, w_full = q_full + 32, w_empty = q_full + 40, o_full = q_full + 48,
                  o_empty = q_full + 56, drain = q_full + 64, st_ready = q_full + 72, st_used = q_full + 80,
                  r_full = q_full + 88, r_used = q_full + 96, never = q_full + 104;
+  // barriers of sketch accumulator ob
+  auto o_full_of = [&](int ob) { return ob ? q_full + 112 : o_full; };
+  auto o_empty_of = [&](int ob) { return ob ? q_full + 120 : o_empty; };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
   volatile uint32_t* skip_flag = reinterpret_cast<volatile uint32_t*>(smem + C::OFF_MISC + 8);
@@ -129,6 +135,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(w_empty, 1);
     mbar_init(o_full, 1);
     mbar_init(o_empty, kSoftWarps);
+    mbar_init(q_full + 112, 1);
+    mbar_init(q_full + 120, kSoftWarps);
     mbar_init(drain, 1);
     // pair mode: st_ready = both warpgroups' partials are in (8 warps; st_used
     // is unused); r_full = the peer's pair has landed (one local expect_tx +
@@ -282,12 +290,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = int(e % C::NSLOT);
         ok = mbar_wait(ring_full(s), (e / C::NSLOT) & 1, abort_flag, a.ws, 0x207);
         if (!ok) break;
-        if (cur.seg_first && sc > 0) {
-          ok = mbar_wait(o_empty, (sc - 1) & 1, abort_flag, a.ws, 0x208);
+        // segment sc accumulates into buffer sc % NOB, free once the softmax
+        // warps have stored the segment that used it last
+        const int ob = sc % C::NOB;
+        if (cur.seg_first && sc >= C::NOB) {
+          ok = mbar_wait(o_empty_of(ob), uint32_t((sc / C::NOB) - 1) & 1u, abort_flag, a.ws, 0x208);
           if (!ok) break;
         }
         tc_fence_after();
         const uint32_t vaddr = sRing + s * C::KV_TILE;
+        const uint32_t ocol = tmem + C::O_COL + uint32_t(ob * C::O_COLS);
 #pragma unroll
         for (int k = 0; k < T / 16; ++k) {
           const uint32_t acc = (cur.seg_first && k == 0) ? 0u : 1u;
@@ -295,14 +307,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             // O^T[d, p] += sum_t V[t, d] A[t, p]:  A-operand V^T (MN-major), B-operand A (MN-major)
             const uint64_t ad = sdesc(vaddr + k * 2048, T * 128, 1024);
             const uint64_t bd = sdesc(sW + k * 2048, T * 128, 1024);
-            umma_ss(tmem + C::O_COL, ad, bd, idO, acc);
+            umma_ss(ocol, ad, bd, idO, acc);
           } else {
 #pragma unroll
             for (int mb = 0; mb < PS / 128; ++mb) {
               // O[p, d] += sum_t A[t, p] V[t, d]: A-operand A^T (MN-major), B-operand V (MN-major)
               const uint64_t ad = sdesc(sW + mb * 2 * (T * 128) + k * 2048, T * 128, 1024);
               const uint64_t bd = sdesc(vaddr + k * 2048, T * 128, 1024);
-              umma_ss(tmem + C::O_COL + mb * D, ad, bd, idO, acc);
+              umma_ss(ocol + mb * D, ad, bd, idO, acc);
             }
           }
         }
@@ -310,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         umma_commit(ring_empty(s));
         ++e;
         if (cur.seg_last) {
-          umma_commit(o_full);
+          umma_commit(o_full_of(ob));
           ++sc;
         }
         cur.next();
@@ -337,6 +349,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       // every wait result is made warp-uniform so a timeout never splits a warp
       auto wwait = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return __all_sync(0xffffffffu, mbar_wait(bar, par, abort_flag, a.ws, site));
+      };
+      // sketch of segment seg_idx (accumulator seg_idx % NOB) waiting to be stored
+      float* pend_dst = nullptr;
+      auto store_pending = [&]() -> bool {
+        const int ob = seg_idx % C::NOB;
+        ok = wwait(o_full_of(ob), uint32_t(seg_idx / C::NOB) & 1u, 0x303);
+        if (!ok) return false;
+        tc_fence_after();
+        store_sketch<D, PS, C::TRANS, C::O_COL>(tmem + uint32_t(ob * C::O_COLS), lane_off, sw, q, lane, pend_dst);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(o_empty_of(ob));
+        ++seg_idx;
+        pend_dst = nullptr;
+        return true;
       };
       // pair mode: the peer's R buffer (second half of the stats area) and
       // its barriers, as shared::cluster addresses
@@ -457,21 +484,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(w_full);
         lse_cur = lse_nxt;
+        // the segment that ended with the previous tile is stored now, after this
+        // tile's weights, so its last aggregation has had a tile's time to finish
+        if (pend_dst != nullptr) {
+          if (!store_pending()) break;
+        }
         if (cur.seg_last) {
-          ok = wwait(o_full, seg_idx & 1, 0x303);
-          if (!ok) break;
-          tc_fence_after();
           const bool whole = cur.seg0 >= tb && cur.seg1 <= te;
-          float* dst = whole ? sketch + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D
-                             : a.partial + ((int64_t(wk) * 2 + partial_slot(total, W, wk, cur.seg0)) * a.P + p0) * D;
-          store_sketch<D, PS, C::TRANS, C::O_COL>(tmem, lane_off, sw, q, lane, dst);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(o_empty);
-          ++seg_idx;
+          pend_dst = whole ? sketch + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D
+                           : a.partial + ((int64_t(wk) * 2 + partial_slot(total, W, wk, cur.seg0)) * a.P + p0) * D;
         }
         cur.next();
       }
+      if (ok && pend_dst != nullptr) store_pending();
     }
   }
   __syncthreads();
