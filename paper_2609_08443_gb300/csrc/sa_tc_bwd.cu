@@ -39,12 +39,15 @@ struct BCfg {
   static constexpr int Q_BYTES = PS * D * 2;
   static constexpr int AB_BYTES = T * PS * 2;
   static constexpr int NSLOT = 4;  // even: even slots hold K tiles, odd slots V tiles
+  static constexpr int NBAR = 2 * NSLOT + 20;
+  // two dsketch buffers where shared memory holds them, so the next user's
+  // dsketch is converted while this user's tiles run
+  static constexpr int NG = (3 * Q_BYTES + AB_BYTES + NSLOT * KV_TILE + NBAR * 8 + 16 <= 232448) ? 2 : 1;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_G = Q_BYTES;
-  static constexpr int OFF_AB = OFF_G + Q_BYTES;
+  static constexpr int OFF_AB = OFF_G + NG * Q_BYTES;
   static constexpr int OFF_RING = OFF_AB + AB_BYTES;
   static constexpr int OFF_BAR = OFF_RING + NSLOT * KV_TILE;
-  static constexpr int NBAR = 2 * NSLOT + 20;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int SMEM = OFF_MISC + 16;
   static constexpr int NSD = (MODE == kSlice) ? 2 : 1;  // S/dA buffers (slice mode has TMEM to spare)
@@ -109,6 +112,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                  sd_free_s = b1 + 40, da_full = b1 + 48, sd_free_da = b1 + 56, a_full = b1 + 64, dv_full = b1 + 72,
                  dv_empty = b1 + 80, ds_full = b1 + 88, ab_empty = b1 + 96, dk_empty = b1 + 104, dq_full = b1 + 112,
                  dq_empty = b1 + 120, drain = b1 + 128;
+  // barriers of dsketch buffer gb
+  auto g_full_of = [&](int gb) { return gb ? b1 + 136 : g_full; };
+  auto g_empty_of = [&](int gb) { return gb ? b1 + 144 : g_empty; };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
 
@@ -129,6 +135,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_empty, 1);
     mbar_init(g_full, 2);
     mbar_init(g_empty, 1);
+    mbar_init(b1 + 136, 2);
+    mbar_init(b1 + 144, 1);
     mbar_init(s_full, 1);
     mbar_init(sd_free_s, kSoftWarps);
     mbar_init(da_full, 1);
@@ -197,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idQD = idesc_bf16(128, D, 1, 1);       // [proto x d], K = tokens
       TileWalker cur(a, tb, te, T), nxt(a, tb, te, T);
       nxt.next();
-      int hc = 0, gc = 0, hp = 0;
+      int hc = 0, gc = 0, hp = 0, gbuf = 0;
       bool ok = true;
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
@@ -229,9 +237,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int sK = int(eK % C::NSLOT), sV = int(eV % C::NSLOT);
         // ---- dA(i) = V(i) G^T
         if (cur.seg_first) {
-          wt(g_full, gc & 1, 0x503);
+          gbuf = gc % C::NG;
+          wt(g_full_of(gbuf), uint32_t(gc / C::NG) & 1u, 0x503);
           ++gc;
         }
+        const uint32_t sGc = sG + uint32_t(gbuf * C::Q_BYTES);
         wt(ring_full(sV), (eV / C::NSLOT) & 1, 0x504);
         wt(sd_free_s, li & 1, 0x505);
         if (!ok) break;
@@ -241,7 +251,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < D / 16; ++k)
             umma_ss(tmem + sdcol(li), sdesc(vaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(sG + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
+                    sdesc(sGc + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
         }
         umma_commit(da_full);
         if (MODE == kSlice) umma_commit(ring_empty(sV));
@@ -254,11 +264,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < PS / 16; ++k)
             umma_ss(tmem + C::DV_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(sG + k * 2048, PS * 128, 1024), idTD, k > 0 ? 1u : 0u);
+                    sdesc(sGc + k * 2048, PS * 128, 1024), idTD, k > 0 ? 1u : 0u);
           umma_commit(dv_full);
         }
         if (!ok) break;
-        if (cur.seg_last) umma_commit(g_empty);
+        if (cur.seg_last) umma_commit(g_empty_of(gbuf));
         const bool more = li + 1 < ntiles;
         const bool newhead = more && nxt.qk != cur.qk;
         // ---- S(i+1) before dK/dQ(i) when its buffer and Q allow it
@@ -335,10 +345,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int li = 0; li < ntiles && ok; ++li) {
         if (cur.seg_first) {
-          if (gc > 0) ok = __all_sync(0xffffffffu, mbar_wait(g_empty, (gc - 1) & 1, abort_flag, a.ws, 0x601));
+          const int gb = gc % C::NG;
+          if (gc >= C::NG)
+            ok = __all_sync(0xffffffffu, mbar_wait(g_empty_of(gb), uint32_t((gc / C::NG) - 1) & 1u, abort_flag,
+                                                   a.ws, 0x601));
           if (!ok) break;
           const float* src = dsk + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D;
+          uint8_t* gdst = smem + C::OFF_G + gb * C::Q_BYTES;
           constexpr int CHUNKS = PS * D / 8;
+#pragma unroll 8
           for (int c = t64; c < CHUNKS; c += 64) {
             const int p = c / (D / 8), dd = (c % (D / 8)) * 8;
             const float4 x = *reinterpret_cast<const float4*>(src + int64_t(p) * D + dd);
@@ -349,11 +364,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             pk.z = pack_bf16(y.x, y.y);
             pk.w = pack_bf16(y.z, y.w);
             const int dh = dd >> 6, chunk = (dd & 63) >> 3;
-            *reinterpret_cast<uint4*>(smem + C::OFF_G + dh * PS * 128 + p * 128 + ((chunk ^ (p & 7)) << 4)) = pk;
+            *reinterpret_cast<uint4*>(gdst + dh * PS * 128 + p * 128 + ((chunk ^ (p & 7)) << 4)) = pk;
           }
           fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0) mbar_arrive(g_full);
+          if (lane == 0) mbar_arrive(g_full_of(gb));
           ++gc;
         }
         cur.next();
