@@ -484,15 +484,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(w_full);
         lse_cur = lse_nxt;
-        // the segment that ended with the previous tile is stored now, after this
-        // tile's weights, so its last aggregation has had a tile's time to finish
-        if (pend_dst != nullptr) {
-          if (!store_pending()) break;
-        }
+        // two accumulators: the segment that ended with the previous tile is
+        // stored now, after this tile's weights, so its last aggregation has had
+        // a tile's time to finish and the next segment accumulates meanwhile;
+        // one accumulator: the segment is stored when it ends (keeping the
+        // pointer across tiles cost the softmax registers for no gain)
+        if (C::NOB == 2 && pend_dst != nullptr && !store_pending()) break;
         if (cur.seg_last) {
           const bool whole = cur.seg0 >= tb && cur.seg1 <= te;
           pend_dst = whole ? sketch + ((int64_t(cur.b) * a.H + cur.h) * a.P + p0) * D
                            : a.partial + ((int64_t(wk) * 2 + partial_slot(total, W, wk, cur.seg0)) * a.P + p0) * D;
+          if (C::NOB == 1 && !store_pending()) break;
         }
         cur.next();
       }

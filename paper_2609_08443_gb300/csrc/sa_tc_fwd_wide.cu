@@ -66,7 +66,7 @@ struct WCfg {
   static constexpr int OFF_W = OFF_V + NV * KV_TILE;
   static constexpr int OFF_X = OFF_W + W_BYTES;
   static constexpr int OFF_BAR = OFF_X + X_BYTES;
-  static constexpr int NBAR = 2 * NK + 2 * NV + 15;
+  static constexpr int NBAR = 2 * NK + 2 * NV + 16;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;  // TMEM address, abort flag + wait limit, skip flag
   static constexpr int SMEM = OFF_MISC + 16;
   static constexpr bool TRANS = (D == 128);  // O^T = V^T A (d on TMEM lanes)
@@ -138,6 +138,7 @@ __global__ void __launch_bounds__(kWThreads, 1)
   auto x_full = [&](int b) { return b1 + 72 + 8u * b; };
   auto x_free = [&](int b) { return b1 + 88 + 8u * b; };
   auto r_free = [&](int b) { return b1 + 104 + 8u * b; };
+  const uint32_t never = b1 + 120;  // completed by nothing: the forced timeout of a test limit
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
   volatile uint32_t* skip_flag = reinterpret_cast<volatile uint32_t*>(smem + C::OFF_MISC + 8);
@@ -168,6 +169,7 @@ __global__ void __launch_bounds__(kWThreads, 1)
     mbar_init(o_full, 1);
     mbar_init(o_empty, kWSoftWarps);
     mbar_init(drain, 1);
+    mbar_init(never, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(x_full(b), kWSoftWarps + 1);
       mbar_init(x_free(b), kWSoftWarps);
@@ -257,7 +259,10 @@ __global__ void __launch_bounds__(kWThreads, 1)
       constexpr uint32_t idO = C::TRANS ? idesc_bf16(128, C::PS, 1, 1) : idesc_bf16(128, D, 1, 1);
       TileWalker ws_(a, tb, te, T), wo(a, tb, te, T);
       int hc = 0, sc = 0, prev_q = -1;
-      bool ok = true;
+      // under a test limit (sa_set_wait_limit_ns) the issuer first waits for a
+      // barrier nothing completes: the limit runs out and the CTA takes its
+      // abort path (drains, TMEM freed, SA_ERR_TIMEOUT)
+      bool ok = ctl_wait_limit(abort_flag) >= kPollLimitNs || mbar_wait(never, 0, abort_flag, a.ws, 0x220);
       auto wt = [&](uint32_t bar, uint32_t par, uint32_t site) {
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
       };

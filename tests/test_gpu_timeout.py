@@ -18,10 +18,11 @@ pytestmark = pytest.mark.gpu
 SA_ERR_TIMEOUT = 5
 
 
-def test_wait_timeout_is_reported_and_the_next_call_is_clean(cuda_lib):
-    assert binding.sa_main_kernel_name(256, 64, binding.SA_BF16, False).startswith("tc")
-    # about 16 tiles per worker, so the pipelines wait for one another
-    spec = wl.custom([70000, 3000, 0, 81000], H=2, P=256, d=64, dtype=wl.BF16, seed=31, bwd=False)
+@pytest.mark.parametrize("P,d", [(256, 64), (512, 128)], ids=["fused", "cluster-pair"])
+def test_wait_timeout_is_reported_and_the_next_call_is_clean(cuda_lib, P, d):
+    assert binding.sa_main_kernel_name(P, d, binding.SA_BF16, False).startswith("tc")
+    # about 16 tiles per worker at P = 256 (32 per cluster pair at P = 512), so the pipelines wait
+    spec = wl.custom([70000, 3000, 0, 81000], H=2, P=P, d=d, dtype=wl.BF16, seed=31, bwd=False)
     t = wl.host_to_torch(spec, wl.make_host(spec), torch.device("cuda"))
     N, H, d = t["K"].shape
     B = t["cu_seqlens"].numel() - 1
