@@ -528,6 +528,48 @@ def copy_ceiling(h_src, h_dst, d_buf, dev, nbytes):
             "how": "torch copy_ between page-locked host and device memory, CUDA events, best of 3"}
 
 
+class HostArrays:
+    """Page-locked host arrays for the e2e leg: anonymous memory advised onto
+    transparent huge pages (MADV_HUGEPAGE), touched, then registered with
+    cudaHostRegister.  On a GB300 host, page-locked memory on small pages
+    copied at 64-80 GB/s in some passes after other processes had run (a
+    translation cost per page), against 193-211 GB/s on huge pages in the same
+    state.  Falls back to torch's page-locked allocator where the mapping or the
+    advice is refused."""
+
+    def __init__(self):
+        self.maps, self.regs, self.kind = [], [], "thp+cudaHostRegister"
+
+    def empty(self, shape, dtype):
+        import mmap
+
+        import torch
+
+        n = int(np.prod(shape)) * torch.empty((), dtype=dtype).element_size()
+        try:
+            mm = mmap.mmap(-1, max(n, 1), flags=mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS)
+            mm.madvise(mmap.MADV_HUGEPAGE)
+            t = torch.frombuffer(mm, dtype=torch.uint8, count=n).view(dtype).view(shape)
+            t.zero_()  # fault the pages in (huge pages where the kernel grants them)
+            if torch.cuda.cudart().cudaHostRegister(t.data_ptr(), n, 0) != 0:
+                raise OSError("cudaHostRegister failed")
+        except (OSError, ValueError, AttributeError):
+            self.kind = "torch pin_memory"
+            return torch.empty(shape, dtype=dtype, pin_memory=True)
+        self.maps.append(mm)
+        self.regs.append(t)
+        return t
+
+    def release(self):
+        import torch
+
+        torch.cuda.synchronize()
+        for t in self.regs:
+            torch.cuda.cudart().cudaHostUnregister(t.data_ptr())
+        self.regs.clear()
+        self.maps.clear()  # the mappings close once the tensors over them are gone
+
+
 def e2e_run(args, spec, data, dkdv, dev):
     """Same metric through the public API with host buffers: every step hands the
     library page-locked host arrays (K, V, Q, dsketch) and gets the host arrays
@@ -543,7 +585,8 @@ def e2e_run(args, spec, data, dkdv, dev):
     B_all, H, P, d = spec.B, spec.H, spec.P, spec.d
 
     def pinned_need(b):
-        # torch's page-locked allocator rounds each block up to a power of two
+        # K, V in and dK, dV out (bf16), dsketch in and sketch out (fp32); with the
+        # fallback allocator each block is rounded up to a power of two
         n = int(lens[:b].sum())
         sizes = [n * H * d * 2] * 4 + [b * H * P * d * 4] * 2
         return sum(1 << (max(s, 1) - 1).bit_length() for s in sizes)
@@ -554,17 +597,17 @@ def e2e_run(args, spec, data, dkdv, dev):
         B -= 1
     N = int(lens[:B].sum())
     cu = torch.from_numpy(wl.cu_seqlens(lens[:B]))
-    pin = dict(dtype=torch.bfloat16, pin_memory=True)
-    h = {"K": torch.empty((N, H, d), **pin), "V": torch.empty((N, H, d), **pin),
-         "Q": torch.empty((H, P, d), **pin), "dsketch": torch.empty((B, H, P, d), dtype=torch.float32,
-                                                                     pin_memory=True),
-         "cu_seqlens": cu.pin_memory()}
+    ha = HostArrays()
+    bf = torch.bfloat16
+    h = {"K": ha.empty((N, H, d), bf), "V": ha.empty((N, H, d), bf), "Q": torch.empty((H, P, d), dtype=bf,
+                                                                                     pin_memory=True),
+         "dsketch": ha.empty((B, H, P, d), torch.float32), "cu_seqlens": cu.pin_memory()}
     for k in ("K", "V"):
         h[k].copy_(data[k][:N])
     h["Q"].copy_(data["Q"])
     h["dsketch"].copy_(data["dsketch"][:B])
-    outs = (torch.empty((B, H, P, d), dtype=torch.float32, pin_memory=True), torch.empty((N, H, d), **pin),
-            torch.empty((N, H, d), **pin), torch.empty((H, P, d), dtype=torch.float32, pin_memory=True))
+    outs = (ha.empty((B, H, P, d), torch.float32), ha.empty((N, H, d), bf), ha.empty((N, H, d), bf),
+            torch.empty((H, P, d), dtype=torch.float32, pin_memory=True))
     ceiling = copy_ceiling(h["K"], outs[1], dkdv[0], dev, min(4 << 30, h["K"].numel() * 2 // 2))
     lib = binding.load()
     ws = torch.empty(lib.sa_step_host_workspace_size(h["cu_seqlens"].data_ptr(), B, H, P, d, binding.SA_BF16, 0),
@@ -588,7 +631,11 @@ def e2e_run(args, spec, data, dkdv, dev):
         times.append(time.perf_counter() - t0)
     mean = sum(times) / len(times)
     med = statistics.median(times)
+    kind = ha.kind
+    del h, outs
+    ha.release()
     return {"value": N / mean, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "host_memory": kind,
             "sample": f"{B} of the {B_all} users (same shapes), page-locked host arrays in and out through "
                       "sa_sketch_step_host (chunks of 262144 tokens, copies overlapped with the step), wall clock, "
                       f"mean of {n} steps" + ("" if B == B_all else
