@@ -560,6 +560,18 @@ class HostArrays:
         self.regs.append(t)
         return t
 
+    @staticmethod
+    def anon_huge_bytes():
+        """This process's anonymous memory on transparent huge pages (bytes), or None."""
+        try:
+            with open("/proc/self/smaps_rollup") as fh:
+                for line in fh:
+                    if line.startswith("AnonHugePages:"):
+                        return int(line.split()[1]) * 1024
+        except OSError:
+            pass
+        return None
+
     def release(self):
         import torch
 
@@ -598,6 +610,7 @@ def e2e_run(args, spec, data, dkdv, dev):
     N = int(lens[:B].sum())
     cu = torch.from_numpy(wl.cu_seqlens(lens[:B]))
     ha = HostArrays()
+    huge0 = HostArrays.anon_huge_bytes()
     bf = torch.bfloat16
     h = {"K": ha.empty((N, H, d), bf), "V": ha.empty((N, H, d), bf), "Q": torch.empty((H, P, d), dtype=bf,
                                                                                      pin_memory=True),
@@ -608,6 +621,7 @@ def e2e_run(args, spec, data, dkdv, dev):
     h["dsketch"].copy_(data["dsketch"][:B])
     outs = (ha.empty((B, H, P, d), torch.float32), ha.empty((N, H, d), bf), ha.empty((N, H, d), bf),
             torch.empty((H, P, d), dtype=torch.float32, pin_memory=True))
+    huge1 = HostArrays.anon_huge_bytes()
     ceiling = copy_ceiling(h["K"], outs[1], dkdv[0], dev, min(4 << 30, h["K"].numel() * 2 // 2))
     lib = binding.load()
     ws = torch.empty(lib.sa_step_host_workspace_size(h["cu_seqlens"].data_ptr(), B, H, P, d, binding.SA_BF16, 0),
@@ -636,6 +650,7 @@ def e2e_run(args, spec, data, dkdv, dev):
     ha.release()
     return {"value": N / mean, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "host_memory": kind,
+            "host_huge_page_bytes": (huge1 - huge0) if huge0 is not None and huge1 is not None else None,
             "sample": f"{B} of the {B_all} users (same shapes), page-locked host arrays in and out through "
                       "sa_sketch_step_host (chunks of 262144 tokens, copies overlapped with the step), wall clock, "
                       f"mean of {n} steps" + ("" if B == B_all else
