@@ -320,6 +320,18 @@ const char* sa_main_kernel_name(int P, int d, sa_dtype dt, int bwd);
 sa_status sa_plan_host(const int32_t* cu_seqlens_host, int B, int H, int tile, int n_workers,
                        int64_t* begin);
 
+/* The tile sequence as the tensor-core kernels walk it: worker w of n_workers
+ * takes its range [begin[w], begin[w+1]) (sa_plan_host), locates its first
+ * tile by a binary search over the users, steps `tile` tokens at a time inside
+ * a (user, head) segment and finds the next segment's user by a forward scan
+ * over the users (falling back to the search after a run of empty users).
+ * Writes, for every tile t of the batch (t < H * tiles per head <= cap), its
+ * user, head, first token row and token count.  Pure C, no GPU; exported for
+ * tests.  SA_ERR_INVALID_ARG if cap is too small, SA_ERR_BAD_SEQLENS for
+ * invalid offsets. */
+sa_status sa_walk_host(const int32_t* cu_seqlens_host, int B, int H, int tile, int n_workers, int32_t* user,
+                       int32_t* head, int64_t* tok0, int32_t* ntok, int64_t cap);
+
 /* The chunks sa_sketch_step_host forms: users [begin[c], begin[c+1]) are chunk
  * c, for c < *n_chunks; `begin` must hold B + 1 entries. */
 sa_status sa_plan_chunks_host(const int32_t* cu_seqlens_host, int B, int64_t chunk_tokens, int* begin,

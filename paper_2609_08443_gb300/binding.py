@@ -96,6 +96,8 @@ def load() -> ctypes.CDLL:
     lib.sa_plan_chunks_host.restype = i32
     lib.sa_plan_host.argtypes = [vp, i32, i32, i32, i32, vp]
     lib.sa_plan_host.restype = i32
+    lib.sa_walk_host.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp, vp, ctypes.c_int64]
+    lib.sa_walk_host.restype = i32
     _lib = lib
     return lib
 
@@ -508,6 +510,22 @@ class SketchAttention(torch.autograd.Function):
         K, V, cu, Q, lse = ctx.saved_tensors
         dK, dV, dQ = sa_sketch_bwd(K, V, cu, Q, dsketch.contiguous(), ctx.scale, lse=lse)
         return dK, dV, None, dQ.to(Q.dtype), None
+
+
+def sa_walk_host(cu_seqlens_host, H: int, tile: int, n_workers: int):
+    """(user, head, tok0, ntok) of every tile in the order the kernels' workers
+    walk them (C: sa_walk_host; pure C, no GPU)."""
+    import numpy as np
+
+    cu = np.ascontiguousarray(cu_seqlens_host, dtype=np.int32)
+    L = np.diff(cu.astype(np.int64))
+    total = int(np.sum((np.maximum(L, 0) + tile - 1) // tile)) * H
+    out = (np.zeros(max(total, 1), np.int32), np.zeros(max(total, 1), np.int32), np.zeros(max(total, 1), np.int64),
+           np.zeros(max(total, 1), np.int32))
+    st = load().sa_walk_host(cu.ctypes.data, cu.size - 1, H, tile, n_workers, *(o.ctypes.data for o in out),
+                             max(total, 1))
+    _check(st, "sa_walk_host")
+    return tuple(o[:total] for o in out)
 
 
 def sa_sketch(K, V, cu_seqlens, Q, scale: Optional[float] = None):

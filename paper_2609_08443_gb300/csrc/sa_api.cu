@@ -662,4 +662,42 @@ sa_status sa_plan_host(const int32_t* cu, int B, int H, int tile, int n_workers,
   return SA_OK;
 }
 
+sa_status sa_walk_host(const int32_t* cu, int B, int H, int tile, int n_workers, int32_t* user, int32_t* head,
+                       int64_t* tok0, int32_t* ntok, int64_t cap) {
+  if (!cu || !user || !head || !tok0 || !ntok || B < 1 || H < 1 || tile < 1 || n_workers < 1)
+    return SA_ERR_INVALID_ARG;
+  if (cu[0] != 0) return SA_ERR_BAD_SEQLENS;
+  std::vector<int64_t> prefix(size_t(B) + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    const int64_t L = int64_t(cu[b + 1]) - int64_t(cu[b]);
+    if (L < 0) return SA_ERR_BAD_SEQLENS;
+    prefix[size_t(b) + 1] = prefix[size_t(b)] + (L + tile - 1) / tile;
+  }
+  const int64_t tph = prefix[size_t(B)], total = tph * H;
+  if (cap < total) return SA_ERR_INVALID_ARG;
+  // each worker's range as the kernels walk it: the first tile located by the
+  // search, then 128-token steps inside a segment and the forward scan across
+  // segment ends
+  for (int w = 0; w < n_workers; ++w) {
+    const int64_t tb = sa::range_begin(total, n_workers, w), te = sa::range_begin(total, n_workers, w + 1);
+    sa::TileRef r{};
+    for (int64_t t = tb; t < te; ++t) {
+      if (t == tb) {
+        r = sa::locate_tile(t, tph, prefix.data(), cu, B, tile);
+      } else if (t < r.seg1) {
+        r.tok0 += tile;
+        const int64_t left = r.L - (t - r.seg0) * tile;
+        r.n = int(left < tile ? left : tile);
+      } else {
+        r = sa::locate_next_segment(t, r.h, r.b, tph, prefix.data(), cu, B, tile);
+      }
+      user[t] = r.b;
+      head[t] = r.h;
+      tok0[t] = r.tok0;
+      ntok[t] = r.n;
+    }
+  }
+  return SA_OK;
+}
+
 }  // extern "C"

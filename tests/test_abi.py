@@ -91,6 +91,40 @@ def test_plan_host_covers_every_tile_once(lib):
                 assert np.all(sizes >= 0) and sizes.max() - sizes.min() <= 1
 
 
+def _tiles_in_order(lens, H, T):
+    """Every tile of the batch in (head, user, tile) order, written out."""
+    cu = np.concatenate([[0], np.cumsum(lens)])
+    rows = []
+    for h in range(H):
+        for b, L in enumerate(lens):
+            for k in range((L + T - 1) // T):
+                rows.append((b, h, cu[b] + k * T, min(T, L - k * T)))
+    return np.array(rows, dtype=np.int64).reshape(-1, 4)
+
+
+def test_walk_host_matches_the_tile_order(lib):
+    """The kernels' walk over their ranges (search for the first tile, steps
+    inside a segment, forward scan to the next segment's user) gives every tile
+    of the (head, user, tile) order, including across runs of empty users longer
+    than the scan (where it falls back to the search) and users cut across
+    workers."""
+    rng = np.random.default_rng(1)
+    gaps = [0] * 9 + [5, 300, 1]                        # nine empty users in a row, then more
+    cases = [[5], [0, 0, 7], [130, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 129, 0],
+             gaps * 3, [0] * 20 + [1] + [0] * 20 + [256],
+             list(rng.integers(0, 600, size=500)),
+             [int(x) if rng.random() < 0.3 else 0 for x in rng.integers(1, 400, size=300)],
+             [100000] * 2 + [0] * 17 + [1, 127, 128, 129]]
+    for lens in cases:
+        cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        for H in (1, 3):
+            want = _tiles_in_order(lens, H, 128)
+            for W in (1, 5, 152, 777):
+                user, head, tok0, ntok = binding.sa_walk_host(cu, H, 128, W)
+                got = np.stack([user, head, tok0, ntok], axis=1).astype(np.int64)
+                assert got.shape == want.shape and np.array_equal(got, want), (lens[:8], H, W)
+
+
 def test_plan_host_rejects_bad_offsets(lib):
     with pytest.raises(binding.SketchError):
         binding.sa_plan_host(np.array([0, 5, 3], np.int32), 1, 128, 4)
