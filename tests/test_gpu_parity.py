@@ -40,6 +40,19 @@ def test_ragged_fwd_bwd(cuda_lib, P, d, dt, H):
     harness.check_spec(spec, bwd=True)
 
 
+# runs of empty users longer than the kernels' forward scan from one segment to
+# the next (eight users), so the walk falls back to its binary search, between
+# short and long users
+EMPTY_RUNS = [300] + [0] * 20 + [129] + [0] * 9 + [1000, 1] + [0] * 12 + [2049, 0, 0, 5] + [0] * 30 + [128]
+
+
+@pytest.mark.parametrize("P,d,dt,H", [(256, 64, wl.BF16, 2), (512, 128, wl.BF16, 2), (128, 128, wl.BF16, 1),
+                                      (1024, 128, wl.BF16, 1), (64, 64, wl.F32, 1)], ids=lambda x: str(x))
+def test_long_runs_of_empty_users(cuda_lib, P, d, dt, H):
+    spec = wl.custom(EMPTY_RUNS, H=H, P=P, d=d, dtype=dt, seed=3 * P + d)
+    harness.check_spec(spec, bwd=True)
+
+
 @pytest.mark.parametrize("pass_lse", [True, False])
 def test_bwd_with_and_without_saved_lse(cuda_lib, pass_lse):
     spec = wl.custom([513, 77, 0, 1300], H=2, P=256, d=64, dtype=wl.BF16, seed=5)
