@@ -3,18 +3,15 @@
 // tokens, and three streams overlap the host-to-device copy of one chunk, the
 // step on the previous chunk and the device-to-host copy of the one before:
 //
-//   copy-in  : K, V, dsketch rows of chunk c -> staging buffer c % kStages
+//   copy-in  : K, V, dsketch rows of chunk c -> staging buffer c % 2
 //   compute  : sa_sketch_fwd + sa_sketch_bwd on the staging buffer; the chunk's
 //              dQ is added into one fp32 accumulator in chunk order
 //   copy-out : sketch, dK, dV rows of chunk c -> the caller's host arrays
 //
 // A chunk's copy-in waits for the copy-out of the chunk that last used its
-// staging buffer.  Three buffers: with two, the copy-in of chunk c + 2 had to
-// wait for the copy-out of chunk c, so every second chunk's copy-in, step and
-// copy-out ran in series (about 20 % of the copy-bound time lost).  dQ
-// reaches the host after the last chunk.  The caller's stream waits for
-// everything before the call returns, so synchronising it means the host
-// outputs are complete.  With page-locked host arrays the
+// staging buffer.  dQ reaches the host after the last chunk.  The caller's
+// stream waits for everything before the call returns, so synchronising it
+// means the host outputs are complete.  With page-locked host arrays the
 // copies run asynchronously; pageable arrays work but serialise the copies.
 #include <mutex>
 #include <vector>
@@ -33,11 +30,9 @@ __global__ void sticky_error_kernel(const uint32_t* __restrict__ src, uint32_t* 
 
 namespace {
 
-constexpr int kStages = 3;  // staging buffers on the device
-
 struct StepStreams {
   cudaStream_t in = nullptr, cmp = nullptr, out = nullptr;
-  cudaEvent_t entry = nullptr, fin = nullptr, in_done[kStages] = {}, cmp_done[kStages] = {}, out_done[kStages] = {};
+  cudaEvent_t entry = nullptr, fin = nullptr, in_done[2] = {}, cmp_done[2] = {}, out_done[2] = {};
   bool ready = false;
 };
 
@@ -56,7 +51,7 @@ sa_status step_streams(StepStreams** out) {
         cudaStreamCreateWithFlags(&s.out, sf) != cudaSuccess || cudaEventCreateWithFlags(&s.entry, ef) != cudaSuccess ||
         cudaEventCreateWithFlags(&s.fin, ef) != cudaSuccess)
       return SA_ERR_CUDA;
-    for (int i = 0; i < kStages; ++i)
+    for (int i = 0; i < 2; ++i)
       if (cudaEventCreateWithFlags(&s.in_done[i], ef) != cudaSuccess ||
           cudaEventCreateWithFlags(&s.cmp_done[i], ef) != cudaSuccess ||
           cudaEventCreateWithFlags(&s.out_done[i], ef) != cudaSuccess)
@@ -98,7 +93,7 @@ sa_status plan_chunks(const int32_t* cu, int B, int64_t chunk_tokens, int max_us
 
 // Device workspace of the pipeline, for chunks of at most Bc users and Nc tokens.
 struct StepLayout {
-  size_t q, dq, cu, stage[kStages], total;
+  size_t q, dq, cu, stage[2], total;
   size_t k, v, g, sk, lse, dk, dv, dqc, ws;  // offsets inside one staging buffer
   size_t stage_bytes, ws_bytes;
 };
@@ -134,8 +129,9 @@ StepLayout step_layout(int B, int n_chunks, int Bc, int64_t Nc, int H, int P, in
   L.ws_bytes = sa_workspace_size(Bc, Nc, H, P, d, dt, 1);
   s = sa::align256(s + L.ws_bytes);
   L.stage_bytes = s;
-  for (int i = 0; i < kStages; ++i) L.stage[i] = off + size_t(i) * s;
-  L.total = off + size_t(kStages) * s;
+  L.stage[0] = off;
+  L.stage[1] = off + s;
+  L.total = off + 2 * s;
   return L;
 }
 
@@ -234,12 +230,12 @@ sa_status sa_sketch_step_host(const void* K, const void* V, const int32_t* cu_se
                             S->in));
   int cu_off = 0;
   for (int c = 0; c < nc; ++c) {
-    const int s = c % kStages;
+    const int s = c & 1;
     const int b0 = begin[c], nb = begin[c + 1] - b0;
     const int64_t t0 = cu_seqlens_host[b0], nt = int64_t(cu_seqlens_host[begin[c + 1]]) - t0;
     char* st = base + L.stage[s];
     // copy-in, once the copy-out of chunk c - 2 has released this buffer
-    if (c >= kStages) STEP_CUDA(cudaStreamWaitEvent(S->in, S->out_done[s], 0));
+    if (c >= 2) STEP_CUDA(cudaStreamWaitEvent(S->in, S->out_done[s], 0));
     if (nt > 0) {
       STEP_CUDA(cudaMemcpyAsync(st + L.k, static_cast<const char*>(K) + size_t(t0) * row, size_t(nt) * row,
                                 cudaMemcpyHostToDevice, S->in));

@@ -125,7 +125,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
       tma_prefetch_desc(&tmQ);
-      TileWalker it(a, tb, te, T), pv(a, tb, te, T), pf(a, tb, te, T);
+      TileWalkerSearch it(a, tb, te, T), pv(a, tb, te, T), pf(a, tb, te, T);
       pf.next();
       pf.next();
       int hc = 0, prev_q = -1;
@@ -181,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ------------------------------------------------------ UMMA issuer
       constexpr uint32_t idS = idesc_bf16(128, T, 0, 0);  // Q (K-major) x K^T (K-major)
       constexpr uint32_t idO = idesc_bf16(128, D, 0, 1);  // A (K-major) x V (MN-major)
-      TileWalker cur(a, tb, te, T), nxt(a, tb, te, T);
+      TileWalkerSearch cur(a, tb, te, T), nxt(a, tb, te, T);
       nxt.next();
       uint32_t e = 0;
       int hc = 0, sc = 0;
@@ -274,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int pr = 128 * g + 32 * q + lane;  // prototype within the CTA's slice
       const uint32_t lane_off = uint32_t(32 * q) << 16;
       const float c2 = a.scale * kLog2e;
-      TileWalker cur(a, tb, te, T);
+      TileWalkerSearch cur(a, tb, te, T);
       int seg_idx = 0;
       bool ok = true;
       float msh = 0.f, l = 0.f;  // shift in use (log2 units) and sum of 2^(S c2 - msh) so far
