@@ -291,8 +291,11 @@ uint64_t sa_launch_count(void);
  * anywhere near 2 s; a lower limit exists so that tests can make a wait run
  * out on purpose and check the recovery: the call's kernels stop, drain their
  * copies and tensor-core work still in flight, release their tensor memory,
- * and sa_get_device_error() reports SA_ERR_TIMEOUT.  The limit is copied into
- * each call's workspace when the call is enqueued. */
+ * and sa_get_device_error() reports SA_ERR_TIMEOUT.  Under a limit below
+ * 1 ms the tensor-core forwards first wait on a barrier that nothing
+ * completes, so such a call always times out (a try-wait may otherwise sleep
+ * until its barrier completes and never see a short limit).  The limit is
+ * copied into each call's workspace when the call is enqueued. */
 sa_status sa_set_wait_limit_ns(uint64_t ns);
 
 /* Kernel selection for all later calls in this process: 0 (default) lets each
