@@ -211,13 +211,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         return ok = ok && mbar_wait(bar, par, abort_flag, a.ws, site);
       };
       auto sdcol = [&](int i) { return uint32_t(C::SD_COL + (i % C::NSD) * PS); };
+      // operand descriptors built once and stepped by constant offsets: each
+      // instruction the issuing thread saves shortens the issue of a group (most
+      // groups here are N = 64 or N = 128, a few dozen cycles of work per UMMA)
+      const uint64_t dQk = sdesc(sQ, 16, 1024), dQm = sdesc(sQ, PS * 128, 1024);
+      const uint64_t dABk = sdesc(sAB, 16, 1024), dABm = sdesc(sAB, T * 128, 1024);
+      const uint64_t dRk = sdesc(sRing, 16, 1024), dRm = sdesc(sRing, T * 128, 1024);
+      const uint64_t dGk = sdesc(sG, 16, 1024), dGm = sdesc(sG, PS * 128, 1024);
       // S(i) = K(i) Q^T into an S/dA buffer
       auto issue_S = [&](uint32_t kslot, uint32_t col) {
-        const uint32_t kaddr = sRing + kslot * C::KV_TILE;
+        const uint64_t dK = sdesc_add(dRk, kslot * C::KV_TILE);
 #pragma unroll
         for (int k = 0; k < D / 16; ++k)
-          umma_ss(tmem + col, sdesc(kaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                  sdesc(sQ + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
+          umma_ss(tmem + col, sdesc_add(dK, (k >> 2) * (T * 128) + (k & 3) * 32),
+                  sdesc_add(dQk, (k >> 2) * (PS * 128) + (k & 3) * 32), idSP, k > 0 ? 1u : 0u);
       };
       TileWalker nx2(a, tb, te, T);
       nx2.next();
@@ -241,17 +248,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           wt(g_full_of(gbuf), uint32_t(gc / C::NG) & 1u, 0x503);
           ++gc;
         }
-        const uint32_t sGc = sG + uint32_t(gbuf * C::Q_BYTES);
         wt(ring_full(sV), (eV / C::NSLOT) & 1, 0x504);
         wt(sd_free_s, li & 1, 0x505);
         if (!ok) break;
         tc_fence_after();
+        const uint32_t gofs = uint32_t(gbuf * C::Q_BYTES);  // this segment's dsketch buffer
         {
-          const uint32_t vaddr = sRing + sV * C::KV_TILE;
+          const uint64_t dVk = sdesc_add(dRk, uint32_t(sV) * C::KV_TILE), dG = sdesc_add(dGk, gofs);
 #pragma unroll
           for (int k = 0; k < D / 16; ++k)
-            umma_ss(tmem + sdcol(li), sdesc(vaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(sGc + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024), idSP, k > 0 ? 1u : 0u);
+            umma_ss(tmem + sdcol(li), sdesc_add(dVk, (k >> 2) * (T * 128) + (k & 3) * 32),
+                    sdesc_add(dG, (k >> 2) * (PS * 128) + (k & 3) * 32), idSP, k > 0 ? 1u : 0u);
         }
         umma_commit(da_full);
         if (MODE == kSlice) umma_commit(ring_empty(sV));
@@ -261,10 +268,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (li > 0) wt(dv_empty, (li - 1) & 1, 0x507);
           if (!ok) break;
           tc_fence_after();
+          const uint64_t dG = sdesc_add(dGm, gofs);
 #pragma unroll
           for (int k = 0; k < PS / 16; ++k)
-            umma_ss(tmem + C::DV_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(sGc + k * 2048, PS * 128, 1024), idTD, k > 0 ? 1u : 0u);
+            umma_ss(tmem + C::DV_COL, sdesc_add(dABk, (k >> 2) * (T * 128) + (k & 3) * 32), sdesc_add(dG, k * 2048),
+                    idTD, k > 0 ? 1u : 0u);
           umma_commit(dv_full);
         }
         if (!ok) break;
@@ -299,17 +307,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (MODE == kFull) {
 #pragma unroll
           for (int k = 0; k < PS / 16; ++k)
-            umma_ss(tmem + C::DK_COL, sdesc(sAB + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024),
-                    sdesc(sQ + k * 2048, PS * 128, 1024), idTD, k > 0 ? 1u : 0u);
+            umma_ss(tmem + C::DK_COL, sdesc_add(dABk, (k >> 2) * (T * 128) + (k & 3) * 32), sdesc_add(dQm, k * 2048),
+                    idTD, k > 0 ? 1u : 0u);
         }
         {
-          const uint32_t kaddr = sRing + sK * C::KV_TILE;
+          const uint64_t dKm = sdesc_add(dRm, uint32_t(sK) * C::KV_TILE);
 #pragma unroll
           for (int k = 0; k < T / 16; ++k)
 #pragma unroll
             for (int mb = 0; mb < PS / 128; ++mb)
-              umma_ss(tmem + C::DQ_COL + mb * D, sdesc(sAB + mb * 2 * (T * 128) + k * 2048, T * 128, 1024),
-                      sdesc(kaddr + k * 2048, T * 128, 1024), idQD, (first_of_hp && k == 0) ? 0u : 1u);
+              umma_ss(tmem + C::DQ_COL + mb * D, sdesc_add(dABm, mb * 2 * (T * 128) + k * 2048),
+                      sdesc_add(dKm, k * 2048), idQD, (first_of_hp && k == 0) ? 0u : 1u);
         }
         umma_commit(ab_empty);
         umma_commit(ring_empty(sK));

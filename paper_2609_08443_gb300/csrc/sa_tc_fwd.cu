@@ -242,14 +242,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       // abort path (drains, TMEM freed, SA_ERR_TIMEOUT)
       bool ok = ctl_wait_limit(abort_flag) >= kPollLimitNs || mbar_wait(never, 0, abort_flag, a.ws, 0x200);
       ok = ok && mbar_wait(q_full, 0, abort_flag, a.ws, 0x201);
+      // operand descriptors built once and stepped by constant offsets: the
+      // issuing thread shares its sub-partition with two softmax warps, and each
+      // instruction it saves shortens the issue of a group
+      const uint64_t dQ0 = sdesc(sQ, 16, 1024), dW0 = sdesc(sW, T * 128, 1024);
+      const uint64_t dK0 = sdesc(sRing, 16, 1024), dV0 = sdesc(sRing, T * 128, 1024);
       auto issue_S = [&](uint32_t slot) {
-        const uint32_t kaddr = sRing + slot * C::KV_TILE;
+        const uint64_t dK = sdesc_add(dK0, slot * C::KV_TILE);
 #pragma unroll
-        for (int k = 0; k < D / 16; ++k) {
-          const uint64_t ad = sdesc(kaddr + (k >> 2) * (T * 128) + (k & 3) * 32, 16, 1024);
-          const uint64_t bd = sdesc(sQ + (k >> 2) * (PS * 128) + (k & 3) * 32, 16, 1024);
-          umma_ss(tmem + C::S_COL, ad, bd, idS, k > 0 ? 1u : 0u);
-        }
+        for (int k = 0; k < D / 16; ++k)
+          umma_ss(tmem + C::S_COL, sdesc_add(dK, (k >> 2) * (T * 128) + (k & 3) * 32),
+                  sdesc_add(dQ0, (k >> 2) * (PS * 128) + (k & 3) * 32), idS, k > 0 ? 1u : 0u);
       };
       if (ok) {
         ok = mbar_wait(ring_full(0), 0, abort_flag, a.ws, 0x202);
@@ -298,24 +301,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
         }
         tc_fence_after();
-        const uint32_t vaddr = sRing + s * C::KV_TILE;
+        const uint64_t dV = sdesc_add(dV0, uint32_t(s) * C::KV_TILE);
         const uint32_t ocol = tmem + C::O_COL + uint32_t(ob * C::O_COLS);
 #pragma unroll
         for (int k = 0; k < T / 16; ++k) {
           const uint32_t acc = (cur.seg_first && k == 0) ? 0u : 1u;
           if (C::TRANS) {
             // O^T[d, p] += sum_t V[t, d] A[t, p]:  A-operand V^T (MN-major), B-operand A (MN-major)
-            const uint64_t ad = sdesc(vaddr + k * 2048, T * 128, 1024);
-            const uint64_t bd = sdesc(sW + k * 2048, T * 128, 1024);
-            umma_ss(ocol, ad, bd, idO, acc);
+            umma_ss(ocol, sdesc_add(dV, k * 2048), sdesc_add(dW0, k * 2048), idO, acc);
           } else {
 #pragma unroll
-            for (int mb = 0; mb < PS / 128; ++mb) {
+            for (int mb = 0; mb < PS / 128; ++mb)
               // O[p, d] += sum_t A[t, p] V[t, d]: A-operand A^T (MN-major), B-operand V (MN-major)
-              const uint64_t ad = sdesc(sW + mb * 2 * (T * 128) + k * 2048, T * 128, 1024);
-              const uint64_t bd = sdesc(vaddr + k * 2048, T * 128, 1024);
-              umma_ss(ocol + mb * D, ad, bd, idO, acc);
-            }
+              umma_ss(ocol + mb * D, sdesc_add(dW0, mb * 2 * (T * 128) + k * 2048), sdesc_add(dV, k * 2048), idO,
+                      acc);
           }
         }
         umma_commit(w_empty);
