@@ -436,7 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float2 fin = rank == 0 ? combine(loc, oth) : combine(oth, loc);
             M = fin.x;
             Z = fin.y;
-            f = ex2((m - M) * c2) / Z;
+            f = ex2((m - M) * c2) * rcp_approx(Z);
           } else {
             // exchange (max, sum) with the other warpgroup's thread of this token
             if (li > 0) {
@@ -454,7 +454,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             M = fmaxf(m, o.x);
             const float f_self = ex2((m - M) * c2), f_other = ex2((o.x - M) * c2);
             Z = z * f_self + o.y * f_other;
-            f = f_self / Z;
+            f = f_self * rcp_approx(Z);
           }
           // rows past the tile's tokens get exact zero weights
           scale_row<C::HALF>(v, valid ? f : 0.f);
