@@ -390,8 +390,9 @@ __global__ void __launch_bounds__(kWThreads, 1)
       const float M = fmaxf(fmaxf(fmax3(pp[0].x, pp[1].x, pp[2].x), fmax3(pp[3].x, pp[4].x, pp[5].x)),
                             fmaxf(pp[6].x, pp[7].x));
       float w[C::NPART];  // each partial's sum rescaled to the common maximum, all exponentials independent
+      const float Mc = M * c2;
 #pragma unroll
-      for (int k = 0; k < C::NPART; ++k) w[k] = pp[k].y * ex2((pp[k].x - M) * c2);
+      for (int k = 0; k < C::NPART; ++k) w[k] = pp[k].y * ex2(fmaf(pp[k].x, c2, -Mc));
       const float Z = ((w[0] + w[1]) + (w[2] + w[3])) + ((w[4] + w[5]) + (w[6] + w[7]));  // fixed tree order
       // the partials are consumed (Z depends on every loaded value): the slots
       // of this buffer may be rewritten, locally and by the peer
@@ -403,7 +404,7 @@ __global__ void __launch_bounds__(kWThreads, 1)
       const bool valid = row < cur.n;
       // rows past the tile's tokens get exact zero weights
       const float rz = __frcp_rn(Z);
-      scale_row<C::GP>(v, valid ? ex2((m - M) * c2) * rz : 0.f);
+      scale_row<C::GP>(v, valid ? ex2(fmaf(m, c2, -Mc)) * rz : 0.f);
       // natural log of Z through the log2 unit (Z lies in [1, 512])
       if (rank == 0 && g == 0 && valid && lse_out)
         lse_out[(cur.tok0 + row) * a.H + cur.h] = M * a.scale + __log2f(Z) * 0.6931471805599453f;
