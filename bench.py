@@ -528,6 +528,48 @@ def copy_ceiling(h_src, h_dst, d_buf, dev, nbytes):
             "how": "torch copy_ between page-locked host and device memory, CUDA events, best of 3"}
 
 
+def array_copy_pass(ins, outs, dev, piece=1 << 30):
+    """One plain pass of a step's copies over the very host arrays the e2e leg
+    hands the library: every byte of ``ins`` host-to-device and every byte of
+    ``outs`` device-to-host, the two directions at once on two streams, in
+    pieces of ``piece`` bytes through two device buffers, no kernels.  Its rate
+    is the copy ceiling of the step's pipeline on this host memory; on a GB300
+    host it fell below the 4 GiB ceiling for ~100 GB of arrays after other
+    processes had run.  Best of two passes, CUDA events."""
+    import torch
+
+    bufs = (torch.empty(piece, dtype=torch.uint8, device=dev), torch.empty(piece, dtype=torch.uint8, device=dev))
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+
+    def pieces(t):
+        f = t.reshape(-1).view(torch.uint8)
+        return [f[o:o + piece] for o in range(0, f.numel(), piece)]
+
+    src = [p for t in ins for p in pieces(t)]
+    dst = [p for t in outs for p in pieces(t)]
+    nbytes = sum(p.numel() for p in src + dst)
+
+    def run():
+        torch.cuda.synchronize(dev)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        ev[0].record(s_in)
+        s_out.wait_event(ev[0])
+        with torch.cuda.stream(s_in):
+            for p in src:
+                bufs[0][:p.numel()].copy_(p, non_blocking=True)
+        with torch.cuda.stream(s_out):
+            for p in dst:
+                p.copy_(bufs[1][:p.numel()], non_blocking=True)
+        ev[1].record(s_in)
+        ev[2].record(s_out)
+        torch.cuda.synchronize(dev)
+        return max(ev[0].elapsed_time(ev[1]), ev[0].elapsed_time(ev[2]))
+
+    ms = min(run() for _ in range(2))
+    return {"gbs": nbytes / (ms / 1e3) / 1e9, "ms": ms, "bytes": int(nbytes),
+            "how": "the e2e arrays copied once in and once out (1 GiB pieces, two streams), no kernels, best of 2"}
+
+
 class HostArrays:
     """Page-locked host arrays for the e2e leg: anonymous memory advised onto
     transparent huge pages (MADV_HUGEPAGE), touched, then registered with
@@ -645,6 +687,7 @@ def e2e_run(args, spec, data, dkdv, dev):
         times.append(time.perf_counter() - t0)
     mean = sum(times) / len(times)
     med = statistics.median(times)
+    arrays = array_copy_pass([h[k] for k in ("K", "V", "Q", "dsketch")], list(outs), dev)
     kind = ha.kind
     del h, outs
     ha.release()
@@ -657,7 +700,7 @@ def e2e_run(args, spec, data, dkdv, dev):
                                               f"; host MemAvailable {avail / 2**30:.0f} GiB limits the users"),
             "ms_per_step": mean * 1e3, "ms_per_step_median": med * 1e3, "value_median": N / med,
             "ms_per_step_all": [t * 1e3 for t in times],
-            "copy_gbs": (h2d + d2h) / mean / 1e9, "copy_ceiling": ceiling}
+            "copy_gbs": (h2d + d2h) / mean / 1e9, "copy_ceiling": ceiling, "array_copy": arrays}
 
 
 def main():
