@@ -185,7 +185,9 @@ sa_status sa_sketch_bwd_tokenwise(const void* K, const void* V, const int32_t* c
  *     a longer user is a chunk of its own; at most 1024 users per chunk).  Three
  *     internal streams overlap the host-to-device copy of a chunk, the step on
  *     the previous chunk and the device-to-host copy of the one before, through
- *     two staging buffers in the workspace; dQ is
+ *     two staging buffers in the workspace (a chunk's copy-in waits for the step
+ *     of the chunk that last used its buffer, its step for that chunk's
+ *     copy-out, so that copy-in and copy-out run side by side); dQ is
  *     summed over the chunks in chunk order (bitwise reproducible for a given
  *     chunk_tokens, but not bitwise equal to one sa_sketch_bwd call on the
  *     whole batch: the summation groups differ).

@@ -8,8 +8,13 @@
 //              dQ is added into one fp32 accumulator in chunk order
 //   copy-out : sketch, dK, dV rows of chunk c -> the caller's host arrays
 //
-// A chunk's copy-in waits for the copy-out of the chunk that last used its
-// staging buffer.  dQ reaches the host after the last chunk.  The caller's
+// A staging buffer holds a chunk's inputs (K, V, dsketch) and, apart from
+// them, its outputs and step workspace.  The step is the last reader of the
+// inputs and the copy-out the last reader of the outputs, so a chunk's copy-in
+// waits only for the step of the chunk that last used its buffer, and its step
+// waits for that chunk's copy-out: the copy-in of chunk c + 2 runs beside the
+// copy-out of chunk c, and the copies, not copy + step + copy, set the pace.
+// dQ reaches the host after the last chunk.  The caller's
 // stream waits for everything before the call returns, so synchronising it
 // means the host outputs are complete.  With page-locked host arrays the
 // copies run asynchronously; pageable arrays work but serialise the copies.
@@ -234,8 +239,8 @@ sa_status sa_sketch_step_host(const void* K, const void* V, const int32_t* cu_se
     const int b0 = begin[c], nb = begin[c + 1] - b0;
     const int64_t t0 = cu_seqlens_host[b0], nt = int64_t(cu_seqlens_host[begin[c + 1]]) - t0;
     char* st = base + L.stage[s];
-    // copy-in, once the copy-out of chunk c - 2 has released this buffer
-    if (c >= 2) STEP_CUDA(cudaStreamWaitEvent(S->in, S->out_done[s], 0));
+    // copy-in, once the step of chunk c - 2 has read this buffer's inputs
+    if (c >= 2) STEP_CUDA(cudaStreamWaitEvent(S->in, S->cmp_done[s], 0));
     if (nt > 0) {
       STEP_CUDA(cudaMemcpyAsync(st + L.k, static_cast<const char*>(K) + size_t(t0) * row, size_t(nt) * row,
                                 cudaMemcpyHostToDevice, S->in));
@@ -245,8 +250,10 @@ sa_status sa_sketch_step_host(const void* K, const void* V, const int32_t* cu_se
     STEP_CUDA(cudaMemcpyAsync(st + L.g, dsketch + size_t(b0) * hpd, size_t(nb) * hpd * 4, cudaMemcpyHostToDevice,
                               S->in));
     STEP_CUDA(cudaEventRecord(S->in_done[s], S->in));
-    // the step on the chunk
+    // the step on the chunk, once the copy-out of chunk c - 2 has read this
+    // buffer's outputs
     STEP_CUDA(cudaStreamWaitEvent(S->cmp, S->in_done[s], 0));
+    if (c >= 2) STEP_CUDA(cudaStreamWaitEvent(S->cmp, S->out_done[s], 0));
     const int32_t* cuc = reinterpret_cast<const int32_t*>(base + L.cu) + cu_off;
     float* skc = reinterpret_cast<float*>(st + L.sk);
     float* lsec = reinterpret_cast<float*>(st + L.lse);
